@@ -1,0 +1,124 @@
+/*
+ * kvdro.h -- C ABI of the GB300 Wasserstein-DRO KV-reservation grid evaluator.
+ *
+ * The library evaluates, on one GPU, the worst-case expected reservation cost
+ * of the paper "Robust KV Cache Management for LLM Serving under Output Token
+ * Length Uncertainty" over a grid of
+ *     regimes m (a (c_p, c_w) pair) x classes k x reservations r x multipliers lam x radii eps
+ * and reduces it to a per-(regime, radius, class) reservation.  For class k with
+ * samples x_1..x_N (output lengths in tokens), support [0, L_k] and input
+ * length L_in_k, with eta = r - L_in_k:
+ *
+ *   Q(eta, xi)   = c_p (xi - eta)^+ + c_w (eta - xi)^+                 (Sec. 2.3; App. A Step 1)
+ *   phi_n        = max{ Q(eta,0) - lam x_n, Q(eta,x_n), Q(eta,L) - lam (L - x_n) }
+ *                                                                       (App. A Step 4)
+ *   S(eta, lam)  = (1/N) sum_n phi_n                                   (App. A Step 3)
+ *   cost(eta,eps)= min_j ( lam_j eps + S(eta, lam_j) )                 (App. A eq. app_kantorovich,
+ *                                                                        gamma restricted to the lam grid)
+ *   r*           = argmin_r cost                                        (Sec. 2.4, eq. dro_obj, r block)
+ *   quantiles    = lower empirical quantiles x_(max(1, ceil(q N)))     (Prop. "Critical Fractile
+ *                                                                        Structure", eq. critical_fractile)
+ *
+ * Conventions shared by every entry point
+ *   - Every function returns a kvdro_status.  Nothing is thrown or aborted across the ABI.
+ *   - Argument errors are found on the host before any launch (KVDRO_EINVAL) and leave the
+ *     context unchanged; kvdro_last_error() then describes the error.
+ *   - Work is enqueued on `stream` (a cudaStream_t; NULL = the legacy default stream).
+ *     Asynchronous CUDA errors surface at the next call or at kvdro_sync() (KVDRO_ECUDA).
+ *   - Array arguments marked "host or device" may point to either; the library inspects the
+ *     pointer.  When any such OUTPUT is in host memory the call blocks until it is filled.
+ *     Device outputs are written asynchronously on `stream`.
+ *   - The caller owns every buffer it passes; the library owns only what kvdro_create() and
+ *     kvdro_load_samples() allocate inside the context, and kvdro_destroy() frees that.
+ *   - A context belongs to one device and one host thread at a time.
+ *   - Ties: the minimum over lam and the argmin over r both take the lowest index.
+ */
+#ifndef KVDRO_H
+#define KVDRO_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct kvdro_ctx kvdro_ctx;
+
+typedef enum {
+    KVDRO_OK = 0,
+    KVDRO_EINVAL = -1,   /* bad argument; nothing was launched */
+    KVDRO_ENOMEM = -2,   /* a device or pinned-host allocation failed */
+    KVDRO_ECUDA = -3,    /* a CUDA call failed (message in kvdro_last_error) */
+    KVDRO_ESTATE = -4,   /* call out of order, e.g. eval before samples are loaded */
+    KVDRO_ETIMEOUT = -5  /* a kernel gave up a bounded wait and reported it */
+} kvdro_status;
+
+typedef enum {
+    KVDRO_FP32 = 0,      /* per-term arithmetic in FP32; sums folded into FP64 */
+    KVDRO_FP64 = 1       /* per-term arithmetic and sums in FP64 */
+} kvdro_precision;
+
+/* Create a context on CUDA device `device_ordinal`.  *out receives the handle (NULL on error). */
+int kvdro_create(kvdro_ctx** out, int device_ordinal);
+
+/*
+ * Load the per-class empirical samples (the empirical distribution of Sec. 2.4 and the
+ * Alg. 1 input) and sort them.  Replaces any previously loaded samples.
+ *   K        number of classes, 1 <= K <= 4096.
+ *   offsets  host int64[K+1], CSR offsets: offsets[0] = 0, N_k = offsets[k+1] - offsets[k] >= 1,
+ *            N_k <= 2^31 - 1.
+ *   lengths  host or device int32[offsets[K]], class k's samples at [offsets[k], offsets[k+1]),
+ *            each in [0, L_max[k]] (checked on the device; a violation gives KVDRO_EINVAL).
+ *   L_max    host int32[K], support upper end L_k, 1 <= L_k <= 2^24.
+ *   L_in     host int32[K] input length per class (>= 0, L_in + L_max <= 2^24), or NULL for zeros.
+ * Runs the segmented counting sort and the cumulative count arrays on `stream`, then blocks
+ * until the range check has been read back.
+ */
+int kvdro_load_samples(kvdro_ctx* ctx, int32_t K, const int64_t* offsets, const int32_t* lengths,
+                       const int32_t* L_max, const int32_t* L_in, void* stream);
+
+/*
+ * Lower empirical quantiles of every loaded class: out[k*F + f] = x_(m), the m-th smallest
+ * sample of class k, m = max(1, ceil(fractiles[f] * N_k)) computed in FP64.
+ *   F          1 <= F <= 65536;  fractiles: host double[F], each in [0, 1].
+ *   out        host or device int32[K*F].
+ */
+int kvdro_quantiles(kvdro_ctx* ctx, int32_t F, const double* fractiles, int32_t* out, void* stream);
+
+/*
+ * Evaluate the grid and reduce it.  Element type of S, cost and min_cost is float for
+ * KVDRO_FP32 and double for KVDRO_FP64.
+ *   R, r       host int32[R], 1 <= R <= 2^20; every r must satisfy L_in_k <= r <= L_in_k + L_k for
+ *              every class (the reservation domain of Sec. 2.2).
+ *   NL, lam    host double[NL], finite, >= 0; 1 <= NL <= 256 (FP32) or 128 (FP64).
+ *   E, eps     host double[E], finite, >= 0; 1 <= E <= 64.
+ *   M, c_p,c_w host double[M] each, finite, >= 0; 1 <= M <= 65536.
+ * Outputs (each may be NULL to skip it; host or device):
+ *   S          [M][K][R][NL]  mean supremum S(eta, lam)
+ *   cost       [M][E][K][R]   min over lam of lam*eps + S
+ *   lam_idx    int32 [M][E][K][R]  lowest lam index attaining cost
+ *   r_idx      int32 [M][E][K]     lowest r index attaining min_r cost
+ *   min_cost   [M][E][K]
+ *   fhat       double [M][E][K]    #{x <= r* - L_in} / N  (empirical CDF at the chosen r)
+ */
+int kvdro_eval_grid(kvdro_ctx* ctx, int precision, int32_t R, const int32_t* r, int32_t NL, const double* lam,
+                    int32_t E, const double* eps, int32_t M, const double* c_p, const double* c_w, void* S,
+                    void* cost, int32_t* lam_idx, int32_t* r_idx, void* min_cost, double* fhat, void* stream);
+
+/* Copy the sorted samples (class by class, ascending, int32[offsets[K]]) to `out` (host or device). */
+int kvdro_sorted_samples(const kvdro_ctx* ctx, int32_t* out, void* stream);
+
+/* Wait for the context's device work and report any asynchronous CUDA error or kernel timeout. */
+int kvdro_sync(kvdro_ctx* ctx);
+
+/* Text of the last error on this context ("" if none).  Valid until the next call on ctx. */
+const char* kvdro_last_error(const kvdro_ctx* ctx);
+
+/* Free the context and everything it owns.  NULL is accepted. */
+int kvdro_destroy(kvdro_ctx* ctx);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* KVDRO_H */

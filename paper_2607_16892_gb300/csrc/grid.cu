@@ -1,0 +1,482 @@
+// Grid evaluation of the worst-case reservation cost (the hot path) and its reductions.
+//
+// What is summed.  For class k (samples x_n in [0, L], count N), regime (c_p, c_w), reservation
+// r with eta = r - L_in in [0, L], and multiplier lam >= 0, the per-sample supremum of App. A
+// Step 4 is the maximum of four affine functions of x:
+//   l1 = c_p (x - eta), l2 = c_w (eta - x)            (the two branches of Q(eta, x))
+//   l3 = Q(eta, 0) - lam x = c_w eta - lam x          (sample moved to xi = 0)
+//   l4 = Q(eta, L) - lam (L - x) = c_p (L - eta) - lam (L - x)   (moved to xi = L)
+// Since l3 - l2 = (c_w - lam) x and l4 - l1 = (c_p - lam)(L - x), with x and L - x >= 0:
+//   max(l2, l3) = V(x) = c_w eta - nu x,           nu = min(lam, c_w)
+//   max(l1, l4) = U(x) = c_p (L - eta) - mu (L - x),  mu = min(lam, c_p)
+// so phi = max(U, V) = V + max(W, 0) with W = U - V = kappa x + d,
+//   kappa = mu + nu,   d = (c_p - mu) L - (c_p + c_w) eta.
+// Summing over the class: sum_n phi_n = N c_w eta - nu sum_n x_n + sum_n max(kappa x_n + d, 0).
+// The first two terms are exact from the class's integer sample sum; the kernel evaluates the
+// last one term by term: one fused multiply-add, one max and one add per (sample, cell).
+//
+// Work decomposition.  A CTA owns one (regime m, class k) and a block of RG*TR consecutive r
+// values for the whole lam grid.  Each warp owns a TR x TL tile of (r, lam) cells; its 32 lanes
+// split the class's samples, which stream through a ring of shared-memory chunks filled by TMA
+// bulk copies (cp.async.bulk + mbarrier).  The FP32 path packs two cells per f32x2 instruction.
+// Every chunk, each lane's FP32 partial sums are transposed and reduced across the warp
+// (fixed shuffle order) so that each lane then owns one cell, folded into an FP64 accumulator.
+// The epilogue forms S = (1/N) sum phi, then for every eps the minimum over lam (lowest index),
+// and feeds the argmin over r through a 64-bit atomicMin on (cost, r index) keys.
+#include <float.h>
+#include <math.h>
+
+#include "kvdro_internal.cuh"
+
+namespace kvdro {
+namespace {
+
+typedef unsigned long long u64;
+
+constexpr int kChunk = 2048;      // samples per staged chunk (16 KB of float2)
+constexpr int kStages = 3;        // ring depth
+constexpr int kMaxThreads = 512;  // up to 16 warps per CTA
+constexpr long long kWaitCycles = 4000000000LL;  // ~2 s at 2 GHz: bound on any barrier wait
+
+template <Prec P>
+struct Tile;
+template <>
+struct Tile<Prec::F32> {
+    static constexpr int TR = 2, TL = 16, LOG2V = 5;
+};
+template <>
+struct Tile<Prec::F64> {
+    static constexpr int TR = 2, TL = 8, LOG2V = 4;
+};
+
+// ---------------------------------------------------------------- PTX helpers
+
+__device__ __forceinline__ u64 pk(float lo, float hi) {
+    u64 r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+    return r;
+}
+__device__ __forceinline__ void upk(u64 r, float& lo, float& hi) {
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(r));
+}
+__device__ __forceinline__ u64 ffma2(u64 a, u64 b, u64 c) {
+    u64 r;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
+    return r;
+}
+__device__ __forceinline__ u64 fadd2(u64 a, u64 b) {
+    u64 r;
+    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+    return r;
+}
+// max(w, 0); a NaN operand yields 0 (PTX max returns the non-NaN input).
+__device__ __forceinline__ float relu(float w) {
+    float d;
+    asm("max.f32 %0, %1, 0f00000000;" : "=f"(d) : "f"(w));
+    return d;
+}
+__device__ __forceinline__ double relu(double w) {
+    double d;
+    asm("max.f64 %0, %1, 0d0000000000000000;" : "=d"(d) : "d"(w));
+    return d;
+}
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void fence_mbar_init() { asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory"); }
+__device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+
+// One bulk copy global -> shared, completing on `bar` (bytes and both addresses 16-byte aligned).
+__device__ __forceinline__ void tma_bulk_load(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+                 "l"(src), "r"(bytes), "r"(bar)
+                 : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Wait for phase `parity` of `bar`; gives up after kWaitCycles and returns false.
+__device__ __noinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity) {
+    if (mbar_try(bar, parity)) return true;
+    const long long t0 = clock64();
+    while (!mbar_try(bar, parity)) {
+        if (clock64() - t0 > kWaitCycles) return false;
+    }
+    return true;
+}
+
+// Reduce V per-lane values across the warp so that lane l ends with the warp-wide sum of value
+// index l >> (5 - log2 V): recursive halving over lane bits 4, 3, ..., then butterflies over the
+// remaining low bits.  The order of additions is fixed, so results are deterministic.
+template <typename T, int V, int S>
+struct TransposeStep {
+    static __device__ __forceinline__ void run(T (&v)[V], int lane) {
+        constexpr int n = V * S / 16;  // values still held per lane before this step
+        if constexpr (n >= 2) {
+            constexpr int h = n / 2;
+            const bool up = (lane & S) != 0;
+#pragma unroll
+            for (int p = 0; p < h; p++) {
+                const T send = up ? v[p] : v[p + h];
+                const T keep = up ? v[p + h] : v[p];
+                v[p] = keep + __shfl_xor_sync(0xffffffffu, send, S);
+            }
+        } else {
+            v[0] += __shfl_xor_sync(0xffffffffu, v[0], S);
+        }
+        if constexpr (S > 1) TransposeStep<T, V, S / 2>::run(v, lane);
+    }
+};
+
+template <typename T, int V>
+__device__ __forceinline__ T transpose_reduce(T (&v)[V], int lane) {
+    TransposeStep<T, V, 16>::run(v, lane);
+    return v[0];
+}
+
+struct SmemLayout {
+    size_t ring, full, lam, eps, S, total;
+};
+
+__host__ __device__ inline SmemLayout smem_layout(int RG, int TR, int NLpad, int E) {
+    SmemLayout L;
+    L.ring = 0;
+    L.full = (size_t)kStages * kChunk * sizeof(float2);
+    L.lam = L.full + 8 * kStages;
+    L.eps = L.lam + 8 * (size_t)NLpad;
+    L.S = L.eps + 8 * (size_t)E;
+    L.total = L.S + 8 * (size_t)RG * TR * NLpad;
+    return L;
+}
+
+// ---------------------------------------------------------------- the grid kernel
+
+template <Prec P>
+__global__ void __launch_bounds__(kMaxThreads, 1) k_grid(const GridArgs a) {
+    constexpr int TR = Tile<P>::TR, TL = Tile<P>::TL, V = TR * TL, LOG2V = Tile<P>::LOG2V;
+    extern __shared__ __align__(128) unsigned char smem[];
+    const int NLpad = a.LT * TL;
+    const SmemLayout lay = smem_layout(a.RG, TR, NLpad, a.E);
+    float2* ring = reinterpret_cast<float2*>(smem + lay.ring);
+    u64* full = reinterpret_cast<u64*>(smem + lay.full);
+    double* s_lam = reinterpret_cast<double*>(smem + lay.lam);
+    double* s_eps = reinterpret_cast<double*>(smem + lay.eps);
+    double* s_S = reinterpret_cast<double*>(smem + lay.S);
+
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nwarps = blockDim.x >> 5;
+    int b = blockIdx.x;
+    const int rb = b % a.r_blocks;
+    b /= a.r_blocks;
+    const int k = b % a.K;
+    const int m = a.m0 + b / a.K;
+    const int lt = warp % a.LT, rg = warp / a.LT;
+    const int r_cta0 = rb * a.RG * TR;
+    const int r_local0 = rg * TR;
+
+    for (int i = tid; i < NLpad; i += blockDim.x) s_lam[i] = i < a.NL ? a.lam[i] : 0.0;
+    for (int i = tid; i < a.E; i += blockDim.x) s_eps[i] = a.eps[i];
+
+    const int64_t pbase = a.pair_off[k];
+    const int64_t np = a.pair_off[k + 1] - pbase;  // multiple of kPadSamples
+    const int nchunks = (int)((np + kChunk - 1) / kChunk);
+    const float2* src = a.pairs + pbase;
+    auto issue = [&](int c) {
+        const int s = c % kStages;
+        const int64_t cnt = min((int64_t)kChunk, np - (int64_t)c * kChunk);
+        tma_bulk_load(smem_u32(ring + (size_t)s * kChunk), src + (int64_t)c * kChunk, (uint32_t)(cnt * sizeof(float2)),
+                      smem_u32(&full[s]));
+    };
+    if (tid == 0) {
+        for (int s = 0; s < kStages; s++) mbar_init(smem_u32(&full[s]), 1);
+        fence_mbar_init();
+    }
+    __syncthreads();
+    if (tid == 0)
+        for (int c = 0; c < kStages && c < nchunks; c++) issue(c);
+    int issued = min(kStages, nchunks);  // chunks issued so far (tracked identically by every thread)
+    int consumed = 0;                    // chunk at which the loop stopped
+
+    // Per-cell constants of this warp's tile (identical across its lanes).
+    const double cp = a.cp[m], cw = a.cw[m], Lk = (double)a.L[k];
+    double eta[TR];
+    bool rvalid[TR];
+#pragma unroll
+    for (int i = 0; i < TR; i++) {
+        const int ri = r_cta0 + r_local0 + i;
+        rvalid[i] = ri < a.R;
+        eta[i] = rvalid[i] ? (double)a.r[ri] - (double)a.L_in[k] : 0.0;
+    }
+
+    bool timeout = false;
+    double acc64 = 0.0;  // this lane's cell after the warp transposition
+
+    if constexpr (P == Prec::F32) {
+        u64 kap[TL / 2], dd[TR][TL / 2], acc[TR][TL / 2];
+#pragma unroll
+        for (int jp = 0; jp < TL / 2; jp++) {
+            const int j0 = lt * TL + 2 * jp;
+            const double l0 = s_lam[j0], l1 = s_lam[j0 + 1];
+            const bool v0 = j0 < a.NL, v1 = j0 + 1 < a.NL;
+            const double mu0 = fmin(l0, cp), mu1 = fmin(l1, cp);
+            kap[jp] = pk(v0 ? (float)(mu0 + fmin(l0, cw)) : 0.f, v1 ? (float)(mu1 + fmin(l1, cw)) : 0.f);
+#pragma unroll
+            for (int i = 0; i < TR; i++) {
+                const double d0 = (cp - mu0) * Lk - (cp + cw) * eta[i];
+                const double d1 = (cp - mu1) * Lk - (cp + cw) * eta[i];
+                dd[i][jp] = pk(v0 && rvalid[i] ? (float)d0 : 0.f, v1 && rvalid[i] ? (float)d1 : 0.f);
+                acc[i][jp] = 0ull;
+            }
+        }
+        for (int c = 0; c < nchunks; c++) {
+            const int s = c % kStages;
+            if (!mbar_wait_bounded(smem_u32(&full[s]), (uint32_t)((c / kStages) & 1))) timeout = true;
+            if (!timeout) {
+                const int cnt = (int)min((int64_t)kChunk, np - (int64_t)c * kChunk);
+                const float4* q = reinterpret_cast<const float4*>(ring + (size_t)s * kChunk);
+                const int nq = cnt >> 6;  // float4 (two samples) per lane
+#pragma unroll 2
+                for (int t = 0; t < nq; t++) {
+                    const float4 v = q[lane + 32 * t];
+                    const u64 xa = pk(v.x, v.y), xb = pk(v.z, v.w);
+#pragma unroll
+                    for (int i = 0; i < TR; i++)
+#pragma unroll
+                        for (int jp = 0; jp < TL / 2; jp++) {
+                            float w0, w1;
+                            upk(ffma2(kap[jp], xa, dd[i][jp]), w0, w1);
+                            acc[i][jp] = fadd2(acc[i][jp], pk(relu(w0), relu(w1)));
+                        }
+#pragma unroll
+                    for (int i = 0; i < TR; i++)
+#pragma unroll
+                        for (int jp = 0; jp < TL / 2; jp++) {
+                            float w0, w1;
+                            upk(ffma2(kap[jp], xb, dd[i][jp]), w0, w1);
+                            acc[i][jp] = fadd2(acc[i][jp], pk(relu(w0), relu(w1)));
+                        }
+                }
+                // Fold this chunk's FP32 partials into the FP64 accumulator of the lane's cell.
+                float vals[V];
+#pragma unroll
+                for (int i = 0; i < TR; i++)
+#pragma unroll
+                    for (int jp = 0; jp < TL / 2; jp++) {
+                        upk(acc[i][jp], vals[i * TL + 2 * jp], vals[i * TL + 2 * jp + 1]);
+                        acc[i][jp] = 0ull;
+                    }
+                acc64 += (double)transpose_reduce<float, V>(vals, lane);
+            }
+            consumed = c;
+            if (__syncthreads_or(timeout)) {
+                timeout = true;
+                break;
+            }
+            if (c + kStages < nchunks) {
+                if (tid == 0) {
+                    fence_proxy_async();
+                    issue(c + kStages);
+                }
+                issued = c + kStages + 1;
+            }
+        }
+    } else {
+        double kap[TL], dd[TR][TL], acc[TR][TL];
+#pragma unroll
+        for (int j = 0; j < TL; j++) {
+            const int lj = lt * TL + j;
+            const double l = s_lam[lj];
+            const bool v = lj < a.NL;
+            const double mu = fmin(l, cp);
+            kap[j] = v ? mu + fmin(l, cw) : 0.0;
+#pragma unroll
+            for (int i = 0; i < TR; i++) {
+                dd[i][j] = (v && rvalid[i]) ? (cp - mu) * Lk - (cp + cw) * eta[i] : 0.0;
+                acc[i][j] = 0.0;
+            }
+        }
+        for (int c = 0; c < nchunks; c++) {
+            const int s = c % kStages;
+            if (!mbar_wait_bounded(smem_u32(&full[s]), (uint32_t)((c / kStages) & 1))) timeout = true;
+            if (!timeout) {
+                const int cnt = (int)min((int64_t)kChunk, np - (int64_t)c * kChunk);
+                const float4* q = reinterpret_cast<const float4*>(ring + (size_t)s * kChunk);
+                const int nq = cnt >> 6;
+                for (int t = 0; t < nq; t++) {
+                    const float4 v = q[lane + 32 * t];
+                    const double xa = (double)v.x, xb = (double)v.z;
+#pragma unroll
+                    for (int i = 0; i < TR; i++)
+#pragma unroll
+                        for (int j = 0; j < TL; j++) {
+                            acc[i][j] += relu(fma(kap[j], xa, dd[i][j]));
+                            acc[i][j] += relu(fma(kap[j], xb, dd[i][j]));
+                        }
+                }
+            }
+            consumed = c;
+            if (__syncthreads_or(timeout)) {
+                timeout = true;
+                break;
+            }
+            if (c + kStages < nchunks) {
+                if (tid == 0) {
+                    fence_proxy_async();
+                    issue(c + kStages);
+                }
+                issued = c + kStages + 1;
+            }
+        }
+        if (!timeout) {
+            double vals[V];
+#pragma unroll
+            for (int i = 0; i < TR; i++)
+#pragma unroll
+                for (int j = 0; j < TL; j++) vals[i * TL + j] = acc[i][j];
+            acc64 = transpose_reduce<double, V>(vals, lane);
+        }
+    }
+
+    if (timeout) {
+        // Report, then let every copy this CTA issued land before the CTA's shared memory is released.
+        if (tid == 0) {
+            atomicOr(a.err + 1, kErrTimeout);
+            for (int c = consumed; c < issued; c++)
+                (void)mbar_wait_bounded(smem_u32(&full[c % kStages]), (uint32_t)((c / kStages) & 1));
+        }
+        __syncthreads();
+        return;
+    }
+
+    // S for this lane's cell.
+    {
+        const int cidx = lane >> (5 - LOG2V);
+        const int i = cidx / TL, j = cidx % TL;
+        const int ri = r_cta0 + r_local0 + i, lj = lt * TL + j;
+        const bool owner = (lane & ((1 << (5 - LOG2V)) - 1)) == 0;
+        if (owner && ri < a.R && lj < a.NL) {
+            const double nu = fmin(s_lam[lj], cw);
+            const double Nk = (double)a.N[k];
+            const double eta_i = (double)a.r[ri] - (double)a.L_in[k];
+            const double tot = Nk * cw * eta_i - nu * (double)a.sumx[k] + acc64;
+            const double S = tot / Nk;
+            s_S[(r_local0 + i) * NLpad + lj] = S;
+            if (a.S_out) {
+                const size_t o = (((size_t)m * a.K + k) * a.R + ri) * a.NL + lj;
+                if constexpr (P == Prec::F32) static_cast<float*>(a.S_out)[o] = (float)S;
+                else static_cast<double*>(a.S_out)[o] = S;
+            }
+        }
+    }
+    __syncthreads();
+
+    // Epilogue: for each (r, eps) of the CTA, the minimum over lam (lowest index on ties), the
+    // cost and lam index outputs, and the argmin over r through a 64-bit atomicMin key.
+    const int rl_count = a.RG * TR;
+    for (int p = warp; p < rl_count * a.E; p += nwarps) {
+        const int rl = p / a.E, e = p % a.E;
+        const int ri = r_cta0 + rl;
+        if (ri >= a.R) continue;
+        double best = DBL_MAX;
+        int bj = 0x7fffffff;
+        for (int j = lane; j < a.NL; j += 32) {
+            const double v = __dadd_rn(__dmul_rn(s_lam[j], s_eps[e]), s_S[rl * NLpad + j]);
+            if (v < best) { best = v; bj = j; }
+        }
+#pragma unroll
+        for (int o = 16; o; o >>= 1) {
+            const double ov = __shfl_xor_sync(0xffffffffu, best, o);
+            const int oj = __shfl_xor_sync(0xffffffffu, bj, o);
+            if (ov < best || (ov == best && oj < bj)) { best = ov; bj = oj; }
+        }
+        if (lane == 0) {
+            const size_t row = ((size_t)m * a.E + e) * a.K + k;
+            const size_t o = row * a.R + ri;
+            u64 key;
+            if constexpr (P == Prec::F32) {
+                const float cf = (float)best;
+                if (a.cost_out) static_cast<float*>(a.cost_out)[o] = cf;
+                key = ((u64)__float_as_uint(cf > 0.f ? cf : 0.f) << 32) | (u64)(uint32_t)ri;
+            } else {
+                static_cast<double*>(a.cost_out)[o] = best;
+                // order-preserving for non-negative doubles; keeps 32 mantissa bits, index in the low 20
+                key = ((u64)__double_as_longlong(best > 0.0 ? best : 0.0) & ~0xFFFFFull) | (u64)ri;
+            }
+            if (a.lam_idx_out) a.lam_idx_out[o] = bj;
+            atomicMin(a.keys + row, key);
+        }
+    }
+}
+
+template <Prec P>
+__global__ void k_finalize(const FinalizeArgs a) {
+    const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= (int64_t)a.M * a.E * a.K) return;
+    const int k = (int)(i % a.K);
+    const u64 key = a.keys[i];
+    if (key == ~0ull) {  // no r evaluated (cannot happen for R >= 1); report an invalid index
+        if (a.r_idx) a.r_idx[i] = -1;
+        return;
+    }
+    const int ri = (int)(P == Prec::F32 ? (key & 0xffffffffull) : (key & 0xFFFFFull));
+    if (a.r_idx) a.r_idx[i] = ri;
+    if (a.min_cost) {
+        if constexpr (P == Prec::F32)
+            static_cast<float*>(a.min_cost)[i] = __uint_as_float((uint32_t)(key >> 32));
+        else
+            static_cast<double*>(a.min_cost)[i] = static_cast<const double*>(a.cost)[i * a.R + ri];
+    }
+    if (a.fhat) {
+        const int32_t v = a.r[ri] - a.L_in[k];
+        a.fhat[i] = (double)a.cdf[a.hist_off[k] + v] / (double)a.N[k];
+    }
+}
+
+}  // namespace
+
+int grid_tile_r(Prec p) { return p == Prec::F32 ? Tile<Prec::F32>::TR : Tile<Prec::F64>::TR; }
+int grid_tile_lam(Prec p) { return p == Prec::F32 ? Tile<Prec::F32>::TL : Tile<Prec::F64>::TL; }
+
+size_t grid_smem_bytes(Prec p, int RG, int LT, int E, int NL) {
+    (void)NL;
+    return smem_layout(RG, grid_tile_r(p), LT * grid_tile_lam(p), E).total;
+}
+
+cudaError_t grid_prepare(Prec p) {
+    // the largest layout: 16 warps, 256 lam, 64 eps
+    const size_t mx = smem_layout(8, 2, 256, 64).total + 4096;
+    if (p == Prec::F32) return cudaFuncSetAttribute(k_grid<Prec::F32>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)mx);
+    return cudaFuncSetAttribute(k_grid<Prec::F64>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)mx);
+}
+
+cudaError_t launch_grid(Prec p, const GridArgs& a, int threads, size_t smem, cudaStream_t s) {
+    const int64_t nblocks = (int64_t)a.m_count * a.K * a.r_blocks;
+    if (nblocks <= 0 || nblocks > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
+    if (p == Prec::F32) k_grid<Prec::F32><<<(unsigned)nblocks, threads, smem, s>>>(a);
+    else k_grid<Prec::F64><<<(unsigned)nblocks, threads, smem, s>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_finalize(Prec p, const FinalizeArgs& a, cudaStream_t s) {
+    const int64_t n = (int64_t)a.M * a.E * a.K;
+    const int threads = 256;
+    const unsigned blocks = (unsigned)((n + threads - 1) / threads);
+    if (p == Prec::F32) k_finalize<Prec::F32><<<blocks, threads, 0, s>>>(a);
+    else k_finalize<Prec::F64><<<blocks, threads, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
+}  // namespace kvdro

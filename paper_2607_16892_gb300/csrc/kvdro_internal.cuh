@@ -1,0 +1,91 @@
+// Internal declarations shared by the library's translation units (not part of the ABI).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace kvdro {
+
+// Samples of one class are staged for the grid kernel as (x, x) float pairs so that one
+// 128-bit shared-memory load yields the packed operands of two samples.  Each class region
+// starts on a multiple of kPadSamples and is padded with NaN pairs, which contribute exactly
+// zero to the excess sum (max(NaN, 0) = 0 in PTX max.f32 / max.f64).
+constexpr int kPadSamples = 128;
+
+// Error bits reported by kernels in ctx->d_err[1].
+constexpr int kErrTimeout = 1;
+
+struct SortArgs {
+    const int32_t* lengths;     // caller samples (device), CSR by class
+    const int64_t* offsets;     // [K+1]
+    const int32_t* L;           // [K]
+    const int64_t* hist_off;    // [K+1] start of class k's cumulative-count array (L_k + 1 entries)
+    const int64_t* pair_off;    // [K+1] start of class k's padded pair region
+    const int32_t* hist_blocks; // [K+1] prefix of histogram blocks per class
+    const int32_t* exp_blocks;  // [K+1] prefix of expand blocks per class
+    int32_t* hist;              // [hist_off[K]] counts, then cumulative counts (in place)
+    int64_t* sumx;              // [K] sum of samples per class
+    int32_t* sorted;            // [offsets[K]]
+    float2* pairs;              // [pair_off[K]]
+    int32_t* err;               // [0] += out-of-range samples
+    int32_t K;
+};
+
+// Launchers (sort.cu)
+cudaError_t launch_histogram(const SortArgs& a, int32_t nblocks, cudaStream_t s);
+cudaError_t launch_scan(const SortArgs& a, cudaStream_t s);
+cudaError_t launch_expand(const SortArgs& a, int32_t nblocks, cudaStream_t s);
+cudaError_t launch_gather_quantiles(const int32_t* sorted, const int64_t* offsets, const int32_t* rank, int32_t K,
+                                    int32_t F, int32_t* out, cudaStream_t s);
+
+enum class Prec { F32 = 0, F64 = 1 };
+
+struct GridArgs {
+    const float2* pairs;        // padded (x, x) pairs
+    const int64_t* pair_off;    // [K+1]
+    const int64_t* N;           // [K]
+    const int64_t* sumx;        // [K]
+    const int32_t* L;           // [K]
+    const int32_t* L_in;        // [K]
+    const int32_t* cdf;         // cumulative counts, class k at hist_off[k]
+    const int64_t* hist_off;    // [K+1]
+    const int32_t* r;           // [R]
+    const double* lam;          // [NL]
+    const double* eps;          // [E]
+    const double* cp;           // [M]
+    const double* cw;           // [M]
+    int32_t K, R, NL, E, M;
+    int32_t LT;                 // lam tiles per CTA
+    int32_t RG;                 // r groups per CTA
+    int32_t r_blocks;           // CTAs per (m, k)
+    int32_t m0, m_count;        // regime range covered by this launch
+    void* S_out;                // optional [M][K][R][NL]
+    void* cost_out;             // [M][E][K][R] (caller's, or scratch for FP64 min_cost)
+    int32_t* lam_idx_out;       // optional [M][E][K][R]
+    unsigned long long* keys;   // [M][E][K] argmin keys (initialised to all ones)
+    int32_t* err;               // [1] |= kErrTimeout
+};
+
+struct FinalizeArgs {
+    const unsigned long long* keys;
+    const void* cost;           // FP64: cost buffer to read min_cost from; FP32 unused
+    const int32_t* r;
+    const int32_t* L_in;
+    const int64_t* N;
+    const int32_t* cdf;
+    const int64_t* hist_off;
+    int32_t K, R, E, M;
+    int32_t* r_idx;             // [M][E][K]
+    void* min_cost;             // [M][E][K]
+    double* fhat;               // [M][E][K]
+};
+
+// grid.cu
+int grid_tile_r(Prec p);                      // r values per warp tile
+int grid_tile_lam(Prec p);                    // lam values per warp tile
+size_t grid_smem_bytes(Prec p, int RG, int LT, int E, int NL);
+cudaError_t grid_prepare(Prec p);             // one-time per-device attribute setup
+cudaError_t launch_grid(Prec p, const GridArgs& a, int threads, size_t smem, cudaStream_t s);
+cudaError_t launch_finalize(Prec p, const FinalizeArgs& a, cudaStream_t s);
+
+}  // namespace kvdro

@@ -1,0 +1,188 @@
+"""Python binding of the kvdro C ABI (include/kvdro.h).
+
+Argument marshalling only: every function here converts its arguments to plain
+pointers and sizes and calls the entry point of the same name in
+``_build/libkvdro.so``.  Every step of the computation runs in that library's
+CUDA kernels; there is no CPU or PyTorch path.  If the library is missing or
+cannot be loaded, the first call raises.
+
+Array arguments may be NumPy arrays (host memory) or torch tensors (host or
+CUDA memory); the library itself tells host from device pointers.  Streams may
+be a ``torch.cuda.Stream``, a raw ``cudaStream_t`` integer, or None (the legacy
+default stream).
+"""
+
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+from typing import Any, Optional
+
+import numpy as np
+
+from . import build as _build
+
+KVDRO_OK = 0
+KVDRO_EINVAL = -1
+KVDRO_ENOMEM = -2
+KVDRO_ECUDA = -3
+KVDRO_ESTATE = -4
+KVDRO_ETIMEOUT = -5
+KVDRO_FP32 = 0
+KVDRO_FP64 = 1
+
+_STATUS = {0: "KVDRO_OK", -1: "KVDRO_EINVAL", -2: "KVDRO_ENOMEM", -3: "KVDRO_ECUDA", -4: "KVDRO_ESTATE",
+           -5: "KVDRO_ETIMEOUT"}
+
+# Every entry point declared in include/kvdro.h.
+SYMBOLS = ("kvdro_create", "kvdro_load_samples", "kvdro_quantiles", "kvdro_eval_grid", "kvdro_sorted_samples",
+           "kvdro_sync", "kvdro_last_error", "kvdro_destroy")
+
+_lock = threading.Lock()
+_lib = None
+
+
+class KvdroError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        super().__init__(f"{_STATUS.get(status, status)}: {message}")
+        self.status = status
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def load_library(build_if_missing: bool = True) -> ctypes.CDLL:
+    """Load libkvdro.so (building it with nvcc first if it is absent)."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        path = _build.LIB
+        if not os.path.exists(path):
+            if not build_if_missing:
+                raise RuntimeError(f"kvdro CUDA library not built: {path}")
+            _build.build()
+        lib = ctypes.CDLL(path)
+        P, i32 = ctypes.c_void_p, ctypes.c_int32
+        lib.kvdro_create.restype = ctypes.c_int
+        lib.kvdro_create.argtypes = [ctypes.POINTER(P), ctypes.c_int]
+        lib.kvdro_load_samples.restype = ctypes.c_int
+        lib.kvdro_load_samples.argtypes = [P, i32, P, P, P, P, P]
+        lib.kvdro_quantiles.restype = ctypes.c_int
+        lib.kvdro_quantiles.argtypes = [P, i32, P, P, P]
+        lib.kvdro_eval_grid.restype = ctypes.c_int
+        lib.kvdro_eval_grid.argtypes = [P, ctypes.c_int, i32, P, i32, P, i32, P, i32, P, P, P, P, P, P, P, P, P]
+        lib.kvdro_sorted_samples.restype = ctypes.c_int
+        lib.kvdro_sorted_samples.argtypes = [P, P, P]
+        lib.kvdro_sync.restype = ctypes.c_int
+        lib.kvdro_sync.argtypes = [P]
+        lib.kvdro_last_error.restype = ctypes.c_char_p
+        lib.kvdro_last_error.argtypes = [P]
+        lib.kvdro_destroy.restype = ctypes.c_int
+        lib.kvdro_destroy.argtypes = [P]
+        _lib = lib
+        return lib
+
+
+# ------------------------------------------------------------------ marshalling
+
+_keep: list = []
+
+
+def _ptr(a: Any, dtype=None):
+    """Pointer to the data of a NumPy array or torch tensor (None -> NULL)."""
+    if a is None:
+        return None
+    if isinstance(a, np.ndarray):
+        if dtype is not None and a.dtype != np.dtype(dtype):
+            raise TypeError(f"expected dtype {np.dtype(dtype)}, got {a.dtype}")
+        if not a.flags["C_CONTIGUOUS"]:
+            raise ValueError("array must be C-contiguous")
+        return a.ctypes.data
+    if hasattr(a, "data_ptr"):
+        if dtype is not None:
+            want = np.dtype(dtype).name
+            got = str(a.dtype).replace("torch.", "")
+            if got != want:
+                raise TypeError(f"expected dtype {want}, got {got}")
+        if not a.is_contiguous():
+            raise ValueError("tensor must be contiguous")
+        return a.data_ptr()
+    raise TypeError(f"unsupported array type {type(a)}")
+
+
+def _host(a: Any, dtype) -> np.ndarray:
+    """Small host-side parameter arrays are converted to contiguous NumPy of the ABI dtype."""
+    if hasattr(a, "detach"):
+        a = a.detach().cpu().numpy()
+    return np.ascontiguousarray(np.asarray(a), dtype=dtype)
+
+
+def _stream(s: Any):
+    if s is None:
+        return None
+    if isinstance(s, int):
+        return s
+    if hasattr(s, "cuda_stream"):
+        return s.cuda_stream
+    raise TypeError(f"unsupported stream {type(s)}")
+
+
+def _check(ctx, status: int):
+    if status != KVDRO_OK:
+        msg = load_library().kvdro_last_error(ctx).decode() if ctx else ""
+        raise KvdroError(status, msg)
+
+
+# ------------------------------------------------------------------ entry points
+
+def kvdro_create(device_ordinal: int = 0) -> ctypes.c_void_p:
+    lib = load_library()
+    h = ctypes.c_void_p()
+    st = lib.kvdro_create(ctypes.byref(h), int(device_ordinal))
+    if st != KVDRO_OK:
+        raise KvdroError(st, f"kvdro_create(device={device_ordinal}) failed")
+    return h
+
+
+def kvdro_load_samples(ctx, K: int, offsets, lengths, L_max, L_in=None, stream=None) -> None:
+    off = _host(offsets, np.int64)
+    lm = _host(L_max, np.int32)
+    li = None if L_in is None else _host(L_in, np.int32)
+    _check(ctx, load_library().kvdro_load_samples(ctx, int(K), off.ctypes.data, _ptr(lengths, np.int32), lm.ctypes.data,
+                                                  None if li is None else li.ctypes.data, _stream(stream)))
+
+
+def kvdro_quantiles(ctx, F: int, fractiles, out, stream=None) -> None:
+    fr = _host(fractiles, np.float64)
+    _check(ctx, load_library().kvdro_quantiles(ctx, int(F), fr.ctypes.data, _ptr(out, np.int32), _stream(stream)))
+
+
+def kvdro_eval_grid(ctx, precision: int, R: int, r, NL: int, lam, E: int, eps, M: int, c_p, c_w, S=None, cost=None,
+                    lam_idx=None, r_idx=None, min_cost=None, fhat=None, stream=None) -> None:
+    ft = np.float32 if precision == KVDRO_FP32 else np.float64
+    rr, ll, ee = _host(r, np.int32), _host(lam, np.float64), _host(eps, np.float64)
+    cp, cw = _host(c_p, np.float64), _host(c_w, np.float64)
+    _check(ctx, load_library().kvdro_eval_grid(
+        ctx, int(precision), int(R), rr.ctypes.data, int(NL), ll.ctypes.data, int(E), ee.ctypes.data, int(M),
+        cp.ctypes.data, cw.ctypes.data, _ptr(S, ft), _ptr(cost, ft), _ptr(lam_idx, np.int32), _ptr(r_idx, np.int32),
+        _ptr(min_cost, ft), _ptr(fhat, np.float64), _stream(stream)))
+
+
+def kvdro_sorted_samples(ctx, out, stream=None) -> None:
+    _check(ctx, load_library().kvdro_sorted_samples(ctx, _ptr(out, np.int32), _stream(stream)))
+
+
+def kvdro_sync(ctx) -> None:
+    _check(ctx, load_library().kvdro_sync(ctx))
+
+
+def kvdro_last_error(ctx) -> str:
+    return load_library().kvdro_last_error(ctx).decode()
+
+
+def kvdro_destroy(ctx) -> None:
+    if ctx:
+        load_library().kvdro_destroy(ctx)

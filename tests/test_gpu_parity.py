@@ -1,0 +1,212 @@
+"""CUDA path versus the oracle on small and ragged cases, edge cases and argument errors.
+
+Every call goes through the C ABI (the ctypes binding).  Sizes span several
+warp tiles, several CTAs and several staged sample chunks, with ragged tails in
+N, R and the lam grid.
+"""
+
+import os
+
+import numpy as np
+import pytest
+
+from oracle import oracle as O
+from synth import Workload, random_case, lognormal_workload_k3_n1e3
+from tests.parity import RTOL, compare_full, rel_close
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+from paper_2607_16892_gb300 import kvdro  # noqa: E402
+from paper_2607_16892_gb300.runner import run  # noqa: E402
+
+P = {"fp32": kvdro.KVDRO_FP32, "fp64": kvdro.KVDRO_FP64}
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _need_gpu():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+
+
+def make(samples_per_class, L, r, lam, eps, cp, cw, L_in=None, fractiles=(0.0, 0.5, 0.9, 1.0), name="case"):
+    cls = [np.asarray(c, np.int32) for c in samples_per_class]
+    off = np.zeros(len(cls) + 1, np.int64)
+    off[1:] = np.cumsum([c.size for c in cls])
+    K = len(cls)
+    return Workload(name=name, samples=np.concatenate(cls), offsets=off,
+                    L=np.broadcast_to(np.asarray(L, np.int32), (K,)).copy(),
+                    L_in=np.zeros(K, np.int32) if L_in is None else np.asarray(L_in, np.int32),
+                    r=np.asarray(r, np.int32), lam=np.asarray(lam, np.float64), eps=np.asarray(eps, np.float64),
+                    cp=np.atleast_1d(np.asarray(cp, np.float64)), cw=np.atleast_1d(np.asarray(cw, np.float64)),
+                    fractiles=np.asarray(fractiles, np.float64))
+
+
+@pytest.mark.parametrize("prec", ["fp64", "fp32"])
+@pytest.mark.parametrize("seed", [1, 2, 3])
+def test_random_ragged_cases(prec, seed):
+    w = random_case(seed, K=3, N=(5000, 777, 33), L=(3000, 3000, 3000), R=45, n_lam=37, n_eps=4, M=3,
+                    lam_range=(1e-3, 200.0), eps_max=300.0)
+    gpu = run(w, P[prec])
+    compare_full(w, gpu, O.solve(w), prec)
+
+
+@pytest.mark.parametrize("prec", ["fp64", "fp32"])
+def test_per_class_support_and_input_length(prec):
+    w = random_case(7, K=4, N=(2100, 129, 128, 1), L=(900, 1500, 2000, 1200), L_in=(0, 50, 10, 200), R=33,
+                    n_lam=16, n_eps=3, M=2, integer_costs=True)
+    compare_full(w, run(w, P[prec]), O.solve(w), prec)
+
+
+@pytest.mark.parametrize("prec", ["fp64", "fp32"])
+def test_lognormal_k3_n1e3_full_grid(prec):
+    w = lognormal_workload_k3_n1e3()
+    rep = compare_full(w, run(w, P[prec]), O.solve(w), prec)
+    if prec == "fp64":
+        assert rep["r_idx_exact"] > 0
+
+
+@pytest.mark.parametrize("prec", ["fp64", "fp32"])
+def test_max_lambda_grid_and_single_points(prec):
+    nl = 256 if prec == "fp32" else 128
+    rng = np.random.default_rng(5)
+    w = make([rng.integers(0, 500, 3000), rng.integers(200, 501, 17)], 500, [0, 250, 500],
+             np.logspace(-4, 3, nl), [0.0, 40.0], [15.0, 2.0], [1.0, 0.5])
+    compare_full(w, run(w, P[prec]), O.solve(w), prec)
+    w1 = make([[7]], 10, [3], [0.5], [2.0], 3.0, 1.0, fractiles=[0.0, 1.0])
+    compare_full(w1, run(w1, P[prec]), O.solve(w1), prec)
+
+
+@pytest.mark.parametrize("prec", ["fp64", "fp32"])
+def test_degenerate_inputs(prec):
+    L = 64
+    cases = [
+        make([np.full(300, 20)], L, np.arange(0, L + 1), [0.0, 0.3, 1.0, 5.0], [0.0, 3.0], 4.0, 1.0),  # one value
+        make([np.array([0, 0, L, L, 0])], L, [0, 1, 32, 63, 64], [0.0, 2.0, 9.0], [0.0, 100.0], 4.0, 1.0),  # ends
+        make([np.arange(0, L + 1)], L, np.arange(0, L + 1, 7), [0.5, 2.0], [1.0], 0.0, 1.0),  # c_p = 0
+        make([np.arange(0, L + 1)], L, np.arange(0, L + 1, 7), [0.5, 2.0], [1.0], 3.0, 0.0),  # c_w = 0
+        make([np.arange(3, 40)], L, [10, 20, 30], [0.0], [0.0, 5.0], 2.0, 1.0),  # lam = 0 only
+    ]
+    for w in cases:
+        compare_full(w, run(w, P[prec]), O.solve(w), prec)
+
+
+def test_worked_example_values():
+    import json
+    g = json.load(open(os.path.join(os.path.dirname(__file__), "golden", "worked_example_n3_L10.json")))
+    w = make([g["samples"]], g["L"], g["r"], g["lam"], g["eps"], g["cp"], g["cw"], fractiles=g["fractiles"])
+    out = run(w, kvdro.KVDRO_FP64)
+    np.testing.assert_allclose(out["S"][0, 0], g["S"], rtol=1e-13)
+    np.testing.assert_allclose(out["cost"][0, :, 0], g["cost"], rtol=1e-13)
+    assert out["lam_idx"][0, :, 0].tolist() == g["lam_idx"]
+    assert out["r_idx"][0, :, 0].tolist() == g["r_idx"]
+    assert out["quant"][0].tolist() == g["quant"]
+    np.testing.assert_allclose(out["fhat"][0, :, 0], g["fhat"], rtol=0)
+
+
+@pytest.mark.parametrize("prec", ["fp64", "fp32"])
+def test_host_buffers_match_device_buffers(prec):
+    w = random_case(21, K=2, N=(3000, 211), L=(700, 700), R=19, n_lam=20, n_eps=2, M=2)
+    a = run(w, P[prec])
+    b = run(w, P[prec], host_outputs=True)
+    for k in a:
+        assert np.array_equal(a[k], b[k]), k
+
+
+def test_repeatable_bit_for_bit():
+    w = random_case(22, K=2, N=(9000, 300), L=(2000, 2000), R=40, n_lam=50, n_eps=3, M=2)
+    a = run(w, kvdro.KVDRO_FP32)
+    b = run(w, kvdro.KVDRO_FP32)
+    for k in a:
+        assert np.array_equal(a[k], b[k]), k
+
+
+def test_reload_and_reuse_context():
+    ctx = kvdro.kvdro_create(0)
+    try:
+        for seed in (31, 32):
+            w = random_case(seed, K=2, N=(1000 + seed, 50), L=(400, 400), R=11, n_lam=9, n_eps=2, M=1)
+            compare_full(w, run(w, kvdro.KVDRO_FP64, ctx=ctx), O.solve(w), "fp64")
+    finally:
+        kvdro.kvdro_destroy(ctx)
+
+
+# ------------------------------------------------------------------ argument errors
+
+def _loaded_ctx():
+    ctx = kvdro.kvdro_create(0)
+    s = torch.tensor([1, 2, 3, 4, 5], dtype=torch.int32, device="cuda")
+    kvdro.kvdro_load_samples(ctx, 1, np.array([0, 5]), s, np.array([10]))
+    return ctx
+
+
+def _status(fn, *a, **kw):
+    try:
+        fn(*a, **kw)
+    except kvdro.KvdroError as e:
+        return e.status
+    return kvdro.KVDRO_OK
+
+
+def test_invalid_arguments_are_rejected_on_the_host():
+    ctx = kvdro.kvdro_create(0)
+    try:
+        ev = lambda **kw: kvdro.kvdro_eval_grid(ctx, kvdro.KVDRO_FP32, 1, [1], 1, [1.0], 1, [0.0], 1, [2.0], [1.0], **kw)
+        assert _status(ev) == kvdro.KVDRO_ESTATE  # nothing loaded yet
+        s = torch.tensor([1, 2, 3], dtype=torch.int32, device="cuda")
+        assert _status(kvdro.kvdro_load_samples, ctx, 0, np.array([0]), s, np.array([], np.int32)) == kvdro.KVDRO_EINVAL
+        assert _status(kvdro.kvdro_load_samples, ctx, 1, np.array([1, 3]), s, np.array([10])) == kvdro.KVDRO_EINVAL
+        assert _status(kvdro.kvdro_load_samples, ctx, 2, np.array([0, 0, 3]), s, np.array([10, 10])) == kvdro.KVDRO_EINVAL
+        assert _status(kvdro.kvdro_load_samples, ctx, 1, np.array([0, 3]), s, np.array([0])) == kvdro.KVDRO_EINVAL
+    finally:
+        kvdro.kvdro_destroy(ctx)
+    ctx = _loaded_ctx()
+    try:
+        E = kvdro.KVDRO_EINVAL
+        f = kvdro.kvdro_eval_grid
+        assert _status(f, ctx, kvdro.KVDRO_FP32, 1, [11], 1, [1.0], 1, [0.0], 1, [2.0], [1.0]) == E     # r > L
+        assert _status(f, ctx, kvdro.KVDRO_FP32, 1, [-1], 1, [1.0], 1, [0.0], 1, [2.0], [1.0]) == E     # r < L_in
+        assert _status(f, ctx, kvdro.KVDRO_FP32, 1, [3], 1, [-1.0], 1, [0.0], 1, [2.0], [1.0]) == E     # lam < 0
+        assert _status(f, ctx, kvdro.KVDRO_FP32, 1, [3], 1, [1.0], 1, [np.nan], 1, [2.0], [1.0]) == E   # eps NaN
+        assert _status(f, ctx, kvdro.KVDRO_FP32, 1, [3], 1, [1.0], 1, [0.0], 1, [np.inf], [1.0]) == E   # c_p inf
+        assert _status(f, ctx, kvdro.KVDRO_FP64, 1, [3], 129, np.ones(129), 1, [0.0], 1, [2.0], [1.0]) == E  # NL cap
+        assert _status(f, ctx, kvdro.KVDRO_FP32, 1, [3], 257, np.ones(257), 1, [0.0], 1, [2.0], [1.0]) == E  # NL cap
+        assert _status(f, ctx, 7, 1, [3], 1, [1.0], 1, [0.0], 1, [2.0], [1.0]) == E                      # precision
+        q = torch.empty(2, dtype=torch.int32, device="cuda")
+        assert _status(kvdro.kvdro_quantiles, ctx, 2, [0.5, 1.5], q) == E
+        # the context still works after rejected calls
+        out = torch.empty(1, dtype=torch.int32, device="cuda")
+        kvdro.kvdro_eval_grid(ctx, kvdro.KVDRO_FP32, 1, [3], 1, [1.0], 1, [0.0], 1, [2.0], [1.0], r_idx=out)
+        kvdro.kvdro_sync(ctx)
+        assert out.item() == 0
+    finally:
+        kvdro.kvdro_destroy(ctx)
+
+
+def test_out_of_range_sample_is_reported_and_unloads():
+    ctx = _loaded_ctx()
+    try:
+        bad = torch.tensor([1, 2, 11, 4], dtype=torch.int32, device="cuda")
+        assert _status(kvdro.kvdro_load_samples, ctx, 1, np.array([0, 4]), bad, np.array([10])) == kvdro.KVDRO_EINVAL
+        assert "outside" in kvdro.kvdro_last_error(ctx)
+        ev = lambda: kvdro.kvdro_eval_grid(ctx, kvdro.KVDRO_FP32, 1, [1], 1, [1.0], 1, [0.0], 1, [2.0], [1.0])
+        assert _status(ev) == kvdro.KVDRO_ESTATE
+        neg = torch.tensor([1, -2], dtype=torch.int32, device="cuda")
+        assert _status(kvdro.kvdro_load_samples, ctx, 1, np.array([0, 2]), neg, np.array([10])) == kvdro.KVDRO_EINVAL
+    finally:
+        kvdro.kvdro_destroy(ctx)
+
+
+def test_injected_allocation_failure_reports_enomem(monkeypatch):
+    for n in (1, 2, 3, 5):
+        monkeypatch.setenv("KVDRO_TEST_FAIL_ALLOC", str(n))
+        ctx = kvdro.kvdro_create(0)
+        try:
+            s = torch.arange(1, 100, dtype=torch.int32, device="cuda")
+            st = _status(kvdro.kvdro_load_samples, ctx, 1, np.array([0, 99]), s, np.array([200]))
+            assert st == kvdro.KVDRO_ENOMEM, n
+        finally:
+            kvdro.kvdro_destroy(ctx)
+    monkeypatch.delenv("KVDRO_TEST_FAIL_ALLOC")
+    ctx = _loaded_ctx()
+    kvdro.kvdro_destroy(ctx)
