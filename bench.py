@@ -1,0 +1,365 @@
+#!/usr/bin/env python3
+"""Throughput of the Wasserstein-DRO reservation-cost path on one GB300 (or N replicas).
+
+One step is one pass of the whole path over the 8-class lognormal workload
+(8 classes x 100,000 samples, 4096 reservations x 128 multipliers x 8 radii,
+c_p/c_w = 10): load + range check + segmented sort of the samples, 5 quantiles,
+the FP32 grid evaluation with its eps epilogue, and the argmin over r.  The
+metric counts one cost term per (class, r, lam, sample) per regime; eps does not
+multiply per-sample work and is not counted.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Under torchrun each rank evaluates its own replica of the workload (independent
+problems, no collective on the data path); the JSON line reports the sum of all
+ranks' terms divided by the slowest rank's time.  ``--impl reference`` times the
+CPU oracle on bounded samples of the same workload instead.
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import re
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from synth import lognormal_workload_k8_n1e5, slice_workload  # noqa: E402
+
+METRIC = "DRO cost terms/sec (class×r×λ×sample) on 1 GB300; % of FP32/HBM roofline"
+UNIT = "terms/s"
+SM_MAX_MHZ_RECIPE = 2070.0
+# Issue bound of the FP32 inner loop: per pair of terms one fma.f32x2, two max.f32 and one
+# add.f32x2 = 4 warp instructions, i.e. 2 issue slots per term; 4 schedulers x 32 lanes per SM.
+TERMS_PER_CLK_PER_SM = 64.0
+GRID_SOURCE = os.path.join(ROOT, "paper_2607_16892_gb300", "csrc", "grid.cu")
+PROFILE = os.path.join(ROOT, "profiles", "k_grid_f32_lognormal_k8_n1e5.md")
+LAUNCHES_PER_STEP = 6  # histogram, scan, expand, quantile gather, grid, argmin finalise
+
+
+def parse_args():
+    p = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=100)
+    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    p.add_argument("--e2e-steps", type=int, default=30)
+    p.add_argument("--cpu-seconds", type=float, default=10.0, help="target wall time of the CPU-baseline sample")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    return p.parse_args()
+
+
+def dist_env():
+    return int(os.environ.get("RANK", 0)), int(os.environ.get("LOCAL_RANK", 0)), int(os.environ.get("WORLD_SIZE", 1))
+
+
+def workload_config(w, world):
+    return {
+        "workload": w.name,
+        "classes": int(w.K),
+        "samples_per_class": int(w.N[0]),
+        "r_points": int(len(w.r)),
+        "lam_points": int(len(w.lam)),
+        "eps_points": int(len(w.eps)),
+        "regimes": int(len(w.cp)),
+        "cost_ratio": float(w.cp[0] / w.cw[0]),
+        "support_L": int(w.L[0]),
+        "fractiles": int(len(w.fractiles)),
+        "terms_per_step_per_gpu": int(w.terms()),
+        "step": "load+range check+segmented sort, quantiles, FP32 grid eval + eps epilogue + argmin over r",
+        "l2": "flushed between timed steps (256 MiB device write outside the timed events)",
+        "parallelism": "single GPU" if world == 1 else f"{world} independent replicas (no data-path collective)",
+    }
+
+
+# ------------------------------------------------------------------ clocks
+
+class ClockSampler:
+    """nvidia-smi clock and throttle-reason samples during the timed region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+    REASONS = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+
+    def __init__(self, gpu_id: str):
+        self.proc = None
+        self.path = None
+        self.gpu_id = gpu_id
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(prefix="kvdro_clocks_", suffix=".csv")
+            os.close(fd)
+            self.fh = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", self.gpu_id, f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=self.fh, stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.fh.close()
+        sm, smax, reasons = [], [], set()
+        for line in open(self.path):
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                smax.append(float(f[2]))
+            except ValueError:
+                continue
+            for name, val in zip(self.REASONS, f[5:9]):
+                if val.lower() == "active":
+                    reasons.add(name)
+        os.unlink(self.path)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ------------------------------------------------------------------ helpers
+
+def reduce_max(value: float, device=None) -> float:
+    """Maximum of a per-rank scalar over all ranks (identity when not distributed)."""
+    import torch
+    import torch.distributed as dist
+
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return value
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def weak_scaling_value(terms_per_rank_step: int, steps: int, world: int, slowest_s: float) -> float:
+    """Whole-job throughput: every rank's terms over the slowest rank's time."""
+    return terms_per_rank_step * steps * world / slowest_s
+
+
+def profile_traffic():
+    """DRAM bytes per grid-kernel launch from the committed ncu summary, if it was taken
+    on the current kernel source (else None)."""
+    try:
+        text = open(PROFILE).read()
+        src_hash = hashlib.sha256(open(GRID_SOURCE, "rb").read()).hexdigest()
+    except OSError:
+        return None
+    m_hash = re.search(r"grid_cu_sha256:\s*([0-9a-f]{64})", text)
+    m_traf = re.search(r"traffic_bytes_per_launch:\s*([0-9.eE+]+)", text)
+    if not m_hash or not m_traf or m_hash.group(1) != src_hash:
+        return None
+    return float(m_traf.group(1))
+
+
+def cpu_baseline(w, seconds: float):
+    """The CPU oracle (direct per-term FP64 evaluation, all host cores) on a bounded,
+    strided slice of the workload's (class, r) rows with the full lam grid and all samples."""
+    from oracle import oracle as O
+
+    threads = O.default_threads()
+    K, R, NL = w.K, len(w.r), len(w.lam)
+
+    def cells_for(rows):
+        ri = np.linspace(0, R - 1, rows).round().astype(np.int64)
+        kk, rr, ll = np.meshgrid(np.arange(K), ri, np.arange(NL), indexing="ij")
+        return np.zeros(kk.size, np.int32), kk.ravel(), rr.ravel(), ll.ravel()
+
+    cal = cells_for(1)
+    t0 = time.perf_counter()
+    O.eval_cells(w, *cal, threads=threads)
+    t_cal = max(time.perf_counter() - t0, 1e-3)
+    rows = int(max(1, min(R, seconds / t_cal)))
+    cells = cells_for(rows)
+    t0 = time.perf_counter()
+    O.eval_cells(w, *cells, threads=threads)
+    dt = time.perf_counter() - t0
+    terms = int(rows * NL * int(w.N.sum()))
+    return {"value": terms / dt, "unit": UNIT, "cores": threads, "kind": "oracle",
+            "sample": f"{rows} strided r rows x {NL} lam x {K} classes x {int(w.N[0])} samples = {terms:.3e} terms, "
+                      f"direct per-term FP64 oracle, {dt:.2f} s wall"}, dt
+
+
+# ------------------------------------------------------------------ our implementation
+
+def run_ours(args):
+    import torch
+
+    rank, local_rank, world = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group(backend="nccl" if torch.cuda.is_available() else "gloo")
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    from paper_2607_16892_gb300 import kvdro as kv
+
+    w = lognormal_workload_k8_n1e5()
+    M, E, K, R, NL, F = len(w.cp), len(w.eps), w.K, len(w.r), len(w.lam), len(w.fractiles)
+    terms = w.terms()
+    ctx = kv.kvdro_create(local_rank)
+    stream = torch.cuda.current_stream(dev)
+    d_samples = torch.from_numpy(w.samples).to(dev)
+    out = {
+        "cost": torch.empty((M, E, K, R), dtype=torch.float32, device=dev),
+        "lam_idx": torch.empty((M, E, K, R), dtype=torch.int32, device=dev),
+        "r_idx": torch.empty((M, E, K), dtype=torch.int32, device=dev),
+        "min_cost": torch.empty((M, E, K), dtype=torch.float32, device=dev),
+        "fhat": torch.empty((M, E, K), dtype=torch.float64, device=dev),
+    }
+    quant = torch.empty((K, F), dtype=torch.int32, device=dev)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+
+    def step(samples, outs, q):
+        kv.kvdro_load_samples(ctx, K, w.offsets, samples, w.L, w.L_in, stream)
+        kv.kvdro_quantiles(ctx, F, w.fractiles, q, stream)
+        kv.kvdro_eval_grid(ctx, kv.KVDRO_FP32, R, w.r, NL, w.lam, E, w.eps, M, w.cp, w.cw, cost=outs["cost"],
+                           lam_idx=outs["lam_idx"], r_idx=outs["r_idx"], min_cost=outs["min_cost"],
+                           fhat=outs["fhat"], stream=stream)
+
+    def barrier():
+        if world > 1:
+            torch.distributed.barrier()
+
+    for _ in range(args.warmup):
+        step(d_samples, out, quant)
+    torch.cuda.synchronize(dev)
+
+    props = torch.cuda.get_device_properties(dev)
+    gpu_id = str(getattr(props, "uuid", local_rank))
+    if gpu_id and not gpu_id.startswith("GPU-") and len(gpu_id) == 36:
+        gpu_id = "GPU-" + gpu_id
+    sampler = ClockSampler(gpu_id)
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    grid_ms = []
+    barrier()
+    torch.cuda.synchronize(dev)
+    sampler.start()
+    wall0 = time.perf_counter()
+    for i in range(args.steps):
+        flush.zero_()  # evict the previous step's data from L2, outside the timed events
+        starts[i].record(stream)
+        step(d_samples, out, quant)
+        ends[i].record(stream)
+        grid_ms.append(kv.kvdro_last_grid_ms(ctx))
+    torch.cuda.synchronize(dev)
+    wall = time.perf_counter() - wall0
+    barrier()
+    clocks = sampler.stop()
+    step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
+    total_s = reduce_max(sum(step_ms) / 1e3, dev)
+    value = weak_scaling_value(terms, args.steps, world, total_s)
+
+    # roofline of the grid kernel (this rank's launches)
+    kernel_ms = statistics.mean(grid_ms)
+    achieved = terms / (kernel_ms / 1e3)
+    peak = props.multi_processor_count * TERMS_PER_CLK_PER_SM * SM_MAX_MHZ_RECIPE * 1e6
+    roofline = {"bound": "alu", "achieved": achieved, "peak": peak, "unit": UNIT, "frac": achieved / peak,
+                "traffic": profile_traffic(), "kernel": "k_grid<F32>",
+                "kernel_ms_mean": kernel_ms,
+                "peak_basis": f"{props.multi_processor_count} SMs x {TERMS_PER_CLK_PER_SM:.0f} terms/clk/SM x "
+                              f"{SM_MAX_MHZ_RECIPE:.0f} MHz (issue bound of the f32x2 inner loop)"}
+    if clocks.get("sm_mhz"):
+        roofline["frac_at_sampled_clock"] = achieved / (peak * clocks["sm_mhz"] / SM_MAX_MHZ_RECIPE)
+
+    # end to end through the C ABI with host buffers: pinned host samples in, host results out
+    h_samples = torch.from_numpy(w.samples).pin_memory()
+    h_out = {k: torch.empty(v.shape, dtype=v.dtype).pin_memory() for k, v in out.items()}
+    h_quant = torch.empty(quant.shape, dtype=quant.dtype).pin_memory()
+    step(h_samples, h_out, h_quant)
+    torch.cuda.synchronize(dev)
+    barrier()
+    t0 = time.perf_counter()
+    for _ in range(args.e2e_steps):
+        step(h_samples, h_out, h_quant)
+    torch.cuda.synchronize(dev)
+    e2e_s = reduce_max(time.perf_counter() - t0, dev)
+    small_in = sum(a.nbytes for a in (w.offsets, w.L, w.L_in, w.r, w.lam, w.eps, w.cp, w.cw, w.fractiles))
+    h2d = int(h_samples.numel() * 4 + small_in)
+    d2h = int(sum(v.numel() * v.element_size() for v in h_out.values()) + h_quant.numel() * 4)
+    e2e = {"value": weak_scaling_value(terms, args.e2e_steps, world, e2e_s), "unit": UNIT, "h2d_bytes_per_step": h2d,
+           "d2h_bytes_per_step": d2h}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu, _ = cpu_baseline(w, args.cpu_seconds)
+
+    kv.kvdro_destroy(ctx)
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": 1e3 * total_s / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": workload_config(w, world), "roofline": roofline, "cpu_baseline": cpu, "e2e": e2e,
+            "clocks": {k: clocks[k] for k in ("sm_mhz", "sm_max_mhz", "reasons")},
+            "gpu_launches": LAUNCHES_PER_STEP * args.steps,
+            "wall_s_timed_region": wall,
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+# ------------------------------------------------------------------ reference arm (the CPU oracle)
+
+def run_reference(args):
+    rank, _, world = dist_env()
+    w = lognormal_workload_k8_n1e5()
+    if rank != 0:
+        return
+    from oracle import oracle as O
+
+    threads = O.default_threads()
+    K, R, NL = w.K, len(w.r), len(w.lam)
+    rows = 2  # per step: 2 strided r rows x all lam x all classes x all samples
+    ri = np.linspace(0, R - 1, rows).round().astype(np.int64)
+    kk, rr, ll = np.meshgrid(np.arange(K), ri, np.arange(NL), indexing="ij")
+    cells = (np.zeros(kk.size, np.int32), kk.ravel(), rr.ravel(), ll.ravel())
+    step_terms = rows * NL * int(w.N.sum())
+    for _ in range(args.warmup):
+        O.eval_cells(w, *cells, threads=threads)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        O.eval_cells(w, *cells, threads=threads)
+    dt = time.perf_counter() - t0
+    value = step_terms * args.steps / dt
+    sample = (f"per step {rows} strided r rows x {NL} lam x {K} classes x {int(w.N[0])} samples = "
+              f"{step_terms:.3e} terms, direct per-term FP64 oracle")
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": workload_config(w, world),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

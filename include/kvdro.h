@@ -108,6 +108,14 @@ int kvdro_eval_grid(kvdro_ctx* ctx, int precision, int32_t R, const int32_t* r, 
 /* Copy the sorted samples (class by class, ascending, int32[offsets[K]]) to `out` (host or device). */
 int kvdro_sorted_samples(const kvdro_ctx* ctx, int32_t* out, void* stream);
 
+/*
+ * Device time, in milliseconds, of the grid-kernel launches of the last kvdro_eval_grid() call on
+ * this context, measured with CUDA events recorded on that call's stream immediately before and
+ * after them (the argmin finalisation and the output copies are outside).  Blocks until the
+ * second event has completed.  KVDRO_ESTATE if no grid has been evaluated yet.
+ */
+int kvdro_last_grid_ms(kvdro_ctx* ctx, float* ms);
+
 /* Wait for the context's device work and report any asynchronous CUDA error or kernel timeout. */
 int kvdro_sync(kvdro_ctx* ctx);
 

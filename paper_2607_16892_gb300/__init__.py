@@ -13,6 +13,7 @@ from .kvdro import (  # noqa: F401
     kvdro_destroy,
     kvdro_eval_grid,
     kvdro_last_error,
+    kvdro_last_grid_ms,
     kvdro_load_samples,
     kvdro_quantiles,
     kvdro_sorted_samples,

@@ -59,6 +59,8 @@ struct kvdro_ctx {
     void* pin = nullptr;  // pinned host staging
     size_t pin_bytes = 0;
     cudaEvent_t pin_free = nullptr;  // completes when the last copy out of `pin` is done
+    cudaEvent_t grid_t0 = nullptr, grid_t1 = nullptr;  // around the last grid-kernel launches
+    bool grid_timed = false;
 
     // device views into `meta`
     int64_t *d_off = nullptr, *d_pair_off = nullptr, *d_hist_off = nullptr, *d_N = nullptr;
@@ -206,7 +208,8 @@ int kvdro_create(kvdro_ctx** out, int device_ordinal) {
     if (const char* f = std::getenv("KVDRO_TEST_FAIL_ALLOC")) ctx->fail_after = std::atoi(f);
     DeviceGuard g(device_ordinal);
     if (!g.ok || kvdro::grid_prepare(Prec::F32) != cudaSuccess || kvdro::grid_prepare(Prec::F64) != cudaSuccess ||
-        cudaEventCreateWithFlags(&ctx->pin_free, cudaEventDisableTiming) != cudaSuccess) {
+        cudaEventCreateWithFlags(&ctx->pin_free, cudaEventDisableTiming) != cudaSuccess ||
+        cudaEventCreate(&ctx->grid_t0) != cudaSuccess || cudaEventCreate(&ctx->grid_t1) != cudaSuccess) {
         cudaGetLastError();
         delete ctx;
         return KVDRO_ECUDA;
@@ -225,6 +228,8 @@ int kvdro_destroy(kvdro_ctx* ctx) {
         release(*b);
     if (ctx->pin) cudaFreeHost(ctx->pin);
     if (ctx->pin_free) cudaEventDestroy(ctx->pin_free);
+    if (ctx->grid_t0) cudaEventDestroy(ctx->grid_t0);
+    if (ctx->grid_t1) cudaEventDestroy(ctx->grid_t1);
     cudaGetLastError();
     delete ctx;
     return KVDRO_OK;
@@ -525,11 +530,15 @@ int kvdro_eval_grid(kvdro_ctx* ctx, int precision, int32_t R, const int32_t* r, 
     a.err = static_cast<int32_t*>(ctx->errs.p);
     const int64_t per_m = (int64_t)ctx->K * r_blocks;
     const int64_t m_step = std::max<int64_t>(1, 0x7fffffffLL / per_m);
+    ctx->grid_timed = false;
+    KV_CUDA(cudaEventRecord(ctx->grid_t0, s), "recording grid start");
     for (int64_t m0 = 0; m0 < M; m0 += m_step) {
         a.m0 = (int32_t)m0;
         a.m_count = (int32_t)std::min<int64_t>(m_step, M - m0);
         KV_CUDA(kvdro::launch_grid(P, a, threads, smem, s), "grid kernel");
     }
+    KV_CUDA(cudaEventRecord(ctx->grid_t1, s), "recording grid end");
+    ctx->grid_timed = true;
 
     kvdro::FinalizeArgs fa;
     fa.keys = static_cast<const unsigned long long*>(ctx->keys.p);
@@ -573,6 +582,17 @@ int kvdro_sorted_samples(const kvdro_ctx* cctx, int32_t* out, void* stream) {
                             dev ? cudaMemcpyDeviceToDevice : cudaMemcpyDeviceToHost, s),
             "copying sorted samples");
     if (!dev) KV_CUDA(cudaStreamSynchronize(s), "copying sorted samples");
+    return KVDRO_OK;
+}
+
+int kvdro_last_grid_ms(kvdro_ctx* ctx, float* ms) {
+    if (!ctx || !ms) return KVDRO_EINVAL;
+    ctx->err.clear();
+    if (!ctx->grid_timed) return fail(ctx, KVDRO_ESTATE, "no grid evaluated yet");
+    DeviceGuard g(ctx->device);
+    if (!g.ok) return fail(ctx, KVDRO_ECUDA, "cannot select device %d", ctx->device);
+    KV_CUDA(cudaEventSynchronize(ctx->grid_t1), "waiting for the grid kernel");
+    KV_CUDA(cudaEventElapsedTime(ms, ctx->grid_t0, ctx->grid_t1), "reading the grid kernel time");
     return KVDRO_OK;
 }
 

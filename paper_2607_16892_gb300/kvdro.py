@@ -37,7 +37,7 @@ _STATUS = {0: "KVDRO_OK", -1: "KVDRO_EINVAL", -2: "KVDRO_ENOMEM", -3: "KVDRO_ECU
 
 # Every entry point declared in include/kvdro.h.
 SYMBOLS = ("kvdro_create", "kvdro_load_samples", "kvdro_quantiles", "kvdro_eval_grid", "kvdro_sorted_samples",
-           "kvdro_sync", "kvdro_last_error", "kvdro_destroy")
+           "kvdro_last_grid_ms", "kvdro_sync", "kvdro_last_error", "kvdro_destroy")
 
 _lock = threading.Lock()
 _lib = None
@@ -76,6 +76,8 @@ def load_library(build_if_missing: bool = True) -> ctypes.CDLL:
         lib.kvdro_eval_grid.argtypes = [P, ctypes.c_int, i32, P, i32, P, i32, P, i32, P, P, P, P, P, P, P, P, P]
         lib.kvdro_sorted_samples.restype = ctypes.c_int
         lib.kvdro_sorted_samples.argtypes = [P, P, P]
+        lib.kvdro_last_grid_ms.restype = ctypes.c_int
+        lib.kvdro_last_grid_ms.argtypes = [P, ctypes.POINTER(ctypes.c_float)]
         lib.kvdro_sync.restype = ctypes.c_int
         lib.kvdro_sync.argtypes = [P]
         lib.kvdro_last_error.restype = ctypes.c_char_p
@@ -173,6 +175,12 @@ def kvdro_eval_grid(ctx, precision: int, R: int, r, NL: int, lam, E: int, eps, M
 
 def kvdro_sorted_samples(ctx, out, stream=None) -> None:
     _check(ctx, load_library().kvdro_sorted_samples(ctx, _ptr(out, np.int32), _stream(stream)))
+
+
+def kvdro_last_grid_ms(ctx) -> float:
+    ms = ctypes.c_float()
+    _check(ctx, load_library().kvdro_last_grid_ms(ctx, ctypes.byref(ms)))
+    return float(ms.value)
 
 
 def kvdro_sync(ctx) -> None:
