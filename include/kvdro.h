@@ -116,6 +116,38 @@ int kvdro_sorted_samples(const kvdro_ctx* ctx, int32_t* out, void* stream);
  */
 int kvdro_last_grid_ms(kvdro_ctx* ctx, float* ms);
 
+/*
+ * kvdro_eval_grid_noalloc -- the FP32 grid evaluation (load, sort, grid, argmin) in one call
+ * that allocates nothing.  The paper has no counterpart; this entry point exists for callers
+ * that cannot allocate device memory at the time they need an answer: a serving engine that
+ * has handed all free device memory to its KV-cache block pool at start-up (a new cudaMalloc
+ * would fail or evict cache blocks), a process held to a fixed device-memory budget, or a
+ * latency-critical loop that must not call cudaMalloc/cudaFree because cudaFree synchronises
+ * the whole device.
+ *
+ * Instead of a context, it works in one static device array of KVDRO_NOALLOC_SCRATCH_BYTES
+ * bytes, defined in the library; every GPU that loads the library holds that array until the
+ * process exits.  The first call on a device (with that device current) resolves the array's
+ * device address and sets a kernel attribute; make that first call before any stream capture.
+ * Calls share the array: it keeps the last call's contents (the call clears what must start at
+ * zero), and calls whose GPU work overlaps in time race on it -- serialise them, e.g. on one
+ * stream.  A problem whose scratch would exceed the array (about 12 bytes per sample plus
+ * 4 bytes per support point and 8 bytes per (regime, radius, class) row) is rejected with
+ * KVDRO_EINVAL and a message.
+ *
+ * Arguments are those of kvdro_load_samples and kvdro_eval_grid with precision KVDRO_FP32,
+ * on the current device, except that `lengths` and every output must be device memory, there
+ * is no S output, and `err` (may be NULL) receives up to err_len bytes of error text.  The
+ * call blocks until the samples' range check is read back; the outputs are written
+ * asynchronously on `stream`.
+ */
+#define KVDRO_NOALLOC_SCRATCH_BYTES (32u << 20)
+int kvdro_eval_grid_noalloc(int32_t K, const int64_t* offsets, const int32_t* lengths, const int32_t* L_max,
+                            const int32_t* L_in, int32_t R, const int32_t* r, int32_t NL, const double* lam,
+                            int32_t E, const double* eps, int32_t M, const double* c_p, const double* c_w,
+                            float* cost, int32_t* lam_idx, int32_t* r_idx, float* min_cost, double* fhat,
+                            void* stream, char* err, int32_t err_len);
+
 /* Wait for the context's device work and report any asynchronous CUDA error or kernel timeout. */
 int kvdro_sync(kvdro_ctx* ctx);
 

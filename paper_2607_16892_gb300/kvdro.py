@@ -37,7 +37,7 @@ _STATUS = {0: "KVDRO_OK", -1: "KVDRO_EINVAL", -2: "KVDRO_ENOMEM", -3: "KVDRO_ECU
 
 # Every entry point declared in include/kvdro.h.
 SYMBOLS = ("kvdro_create", "kvdro_load_samples", "kvdro_quantiles", "kvdro_eval_grid", "kvdro_sorted_samples",
-           "kvdro_last_grid_ms", "kvdro_sync", "kvdro_last_error", "kvdro_destroy")
+           "kvdro_last_grid_ms", "kvdro_eval_grid_noalloc", "kvdro_sync", "kvdro_last_error", "kvdro_destroy")
 
 _lock = threading.Lock()
 _lib = None
@@ -78,6 +78,9 @@ def load_library(build_if_missing: bool = True) -> ctypes.CDLL:
         lib.kvdro_sorted_samples.argtypes = [P, P, P]
         lib.kvdro_last_grid_ms.restype = ctypes.c_int
         lib.kvdro_last_grid_ms.argtypes = [P, ctypes.POINTER(ctypes.c_float)]
+        lib.kvdro_eval_grid_noalloc.restype = ctypes.c_int
+        lib.kvdro_eval_grid_noalloc.argtypes = [i32, P, P, P, P, i32, P, i32, P, i32, P, i32, P, P, P, P, P, P, P, P,
+                                                ctypes.c_char_p, i32]
         lib.kvdro_sync.restype = ctypes.c_int
         lib.kvdro_sync.argtypes = [P]
         lib.kvdro_last_error.restype = ctypes.c_char_p
@@ -181,6 +184,25 @@ def kvdro_last_grid_ms(ctx) -> float:
     ms = ctypes.c_float()
     _check(ctx, load_library().kvdro_last_grid_ms(ctx, ctypes.byref(ms)))
     return float(ms.value)
+
+
+def kvdro_eval_grid_noalloc(K: int, offsets, lengths, L_max, L_in, R: int, r, NL: int, lam, E: int, eps, M: int,
+                            c_p, c_w, cost=None, lam_idx=None, r_idx=None, min_cost=None, fhat=None,
+                            stream=None) -> None:
+    """FP32 grid pass in the library's static scratch (allocates nothing; see include/kvdro.h).
+    ``lengths`` and the outputs must be CUDA tensors on the current device."""
+    off, lm = _host(offsets, np.int64), _host(L_max, np.int32)
+    li = None if L_in is None else _host(L_in, np.int32)
+    rr, ll, ee = _host(r, np.int32), _host(lam, np.float64), _host(eps, np.float64)
+    cp, cw = _host(c_p, np.float64), _host(c_w, np.float64)
+    buf = ctypes.create_string_buffer(512)
+    st = load_library().kvdro_eval_grid_noalloc(
+        int(K), off.ctypes.data, _ptr(lengths, np.int32), lm.ctypes.data, None if li is None else li.ctypes.data,
+        int(R), rr.ctypes.data, int(NL), ll.ctypes.data, int(E), ee.ctypes.data, int(M), cp.ctypes.data,
+        cw.ctypes.data, _ptr(cost, np.float32), _ptr(lam_idx, np.int32), _ptr(r_idx, np.int32),
+        _ptr(min_cost, np.float32), _ptr(fhat, np.float64), _stream(stream), buf, len(buf))
+    if st != KVDRO_OK:
+        raise KvdroError(st, buf.value.decode())
 
 
 def kvdro_sync(ctx) -> None:
