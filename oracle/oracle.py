@@ -177,13 +177,17 @@ def envelope_grid(w, threads: Optional[int] = None) -> np.ndarray:
 def eps_epilogue(S: np.ndarray, lam: np.ndarray, eps: np.ndarray):
     """cost[m, e, k, r] = min_j (lam_j eps_e + S[m, k, r, j]) -- the dual objective of
     App. A (strong duality, gamma restricted to the lam grid); lam_idx is the lowest j
-    attaining the minimum (reading: ties go to the lowest index)."""
+    attaining the minimum (reading: ties go to the lowest index).  One radius at a time."""
     lam = np.asarray(lam, np.float64)
     eps = np.asarray(eps, np.float64)
-    # obj[m, e, k, r, j]
-    obj = lam[None, None, None, None, :] * eps[None, :, None, None, None] + S[:, None, :, :, :]
-    lam_idx = np.argmin(obj, axis=-1).astype(np.int32)       # first occurrence = lowest index
-    cost = np.take_along_axis(obj, lam_idx[..., None].astype(np.int64), axis=-1)[..., 0]
+    M, K, R, NL = S.shape
+    cost = np.empty((M, eps.size, K, R), np.float64)
+    lam_idx = np.empty((M, eps.size, K, R), np.int32)
+    for e, ep in enumerate(eps):
+        obj = lam[None, None, None, :] * ep + S                 # [m, k, r, j]
+        j = np.argmin(obj, axis=-1)                            # first occurrence = lowest index
+        lam_idx[:, e] = j
+        cost[:, e] = np.take_along_axis(obj, j[..., None], axis=-1)[..., 0]
     return cost, lam_idx
 
 

@@ -38,16 +38,20 @@ constexpr int kStages = 3;        // ring depth
 constexpr int kMaxThreads = 512;  // up to 16 warps per CTA
 constexpr long long kWaitCycles = 4000000000LL;  // ~2 s at 2 GHz: bound on any barrier wait
 
-template <Prec P>
-struct Tile;
-template <>
-struct Tile<Prec::F32> {
-    static constexpr int TR = 2, TL = 16, LOG2V = 5;
+constexpr int ilog2(int v) { return v <= 1 ? 0 : 1 + ilog2(v / 2); }
+
+// Shape of one instantiation of the grid kernel: precision, warp tile (TR reservations x TL
+// multipliers, TR*TL a power of two <= 32), FP32 chunks between folds of the per-lane partial
+// sums into FP64 (FP64 folds once at the end), and the minimum CTAs per SM it is built for.
+template <Prec P_, int TR_, int TL_, int FLUSH_, int MINB_>
+struct GridCfg {
+    static constexpr Prec P = P_;
+    static constexpr int TR = TR_, TL = TL_, V = TR_ * TL_, LOG2V = ilog2(TR_ * TL_), FLUSH = FLUSH_, MINB = MINB_;
+    static_assert((V & (V - 1)) == 0 && V >= 2 && V <= 32, "tile must hold a power of two <= 32 cells");
+    static_assert(P_ == Prec::F64 || TL_ % 2 == 0, "the FP32 tile packs lam values in pairs");
 };
-template <>
-struct Tile<Prec::F64> {
-    static constexpr int TR = 2, TL = 8, LOG2V = 4;
-};
+using CfgF32 = GridCfg<Prec::F32, 2, 16, 2, 1>;
+using CfgF64 = GridCfg<Prec::F64, 2, 8, 0, 1>;
 
 // ---------------------------------------------------------------- PTX helpers
 
@@ -165,9 +169,10 @@ __host__ __device__ inline SmemLayout smem_layout(int RG, int TR, int NLpad, int
 
 // ---------------------------------------------------------------- the grid kernel
 
-template <Prec P>
-__global__ void __launch_bounds__(kMaxThreads, 1) k_grid(const GridArgs a) {
-    constexpr int TR = Tile<P>::TR, TL = Tile<P>::TL, V = TR * TL, LOG2V = Tile<P>::LOG2V;
+template <class C>
+__global__ void __launch_bounds__(kMaxThreads, C::MINB) k_grid(const GridArgs a) {
+    constexpr Prec P = C::P;
+    constexpr int TR = C::TR, TL = C::TL, V = C::V, LOG2V = C::LOG2V;
     extern __shared__ __align__(128) unsigned char smem[];
     const int NLpad = a.LT * TL;
     const SmemLayout lay = smem_layout(a.RG, TR, NLpad, a.E);
@@ -269,16 +274,19 @@ __global__ void __launch_bounds__(kMaxThreads, 1) k_grid(const GridArgs a) {
                             acc[i][jp] = fadd2(acc[i][jp], pk(relu(w0), relu(w1)));
                         }
                 }
-                // Fold this chunk's FP32 partials into the FP64 accumulator of the lane's cell.
-                float vals[V];
+                // Every C::FLUSH chunks (and after the last), fold the FP32 partials into the FP64
+                // accumulator of the lane's cell.
+                if ((c + 1) % C::FLUSH == 0 || c + 1 == nchunks) {
+                    float vals[V];
 #pragma unroll
-                for (int i = 0; i < TR; i++)
+                    for (int i = 0; i < TR; i++)
 #pragma unroll
-                    for (int jp = 0; jp < TL / 2; jp++) {
-                        upk(acc[i][jp], vals[i * TL + 2 * jp], vals[i * TL + 2 * jp + 1]);
-                        acc[i][jp] = 0ull;
-                    }
-                acc64 += (double)transpose_reduce<float, V>(vals, lane);
+                        for (int jp = 0; jp < TL / 2; jp++) {
+                            upk(acc[i][jp], vals[i * TL + 2 * jp], vals[i * TL + 2 * jp + 1]);
+                            acc[i][jp] = 0ull;
+                        }
+                    acc64 += (double)transpose_reduce<float, V>(vals, lane);
+                }
             }
             consumed = c;
             if (__syncthreads_or(timeout)) {
@@ -447,8 +455,8 @@ __global__ void k_finalize(const FinalizeArgs a) {
 
 }  // namespace
 
-int grid_tile_r(Prec p) { return p == Prec::F32 ? Tile<Prec::F32>::TR : Tile<Prec::F64>::TR; }
-int grid_tile_lam(Prec p) { return p == Prec::F32 ? Tile<Prec::F32>::TL : Tile<Prec::F64>::TL; }
+int grid_tile_r(Prec p) { return p == Prec::F32 ? CfgF32::TR : CfgF64::TR; }
+int grid_tile_lam(Prec p) { return p == Prec::F32 ? CfgF32::TL : CfgF64::TL; }
 
 size_t grid_smem_bytes(Prec p, int RG, int LT, int E, int NL) {
     (void)NL;
@@ -458,15 +466,15 @@ size_t grid_smem_bytes(Prec p, int RG, int LT, int E, int NL) {
 cudaError_t grid_prepare(Prec p) {
     // the largest layout: 16 warps, 256 lam, 64 eps
     const size_t mx = smem_layout(8, 2, 256, 64).total + 4096;
-    if (p == Prec::F32) return cudaFuncSetAttribute(k_grid<Prec::F32>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)mx);
-    return cudaFuncSetAttribute(k_grid<Prec::F64>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)mx);
+    if (p == Prec::F32) return cudaFuncSetAttribute(k_grid<CfgF32>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)mx);
+    return cudaFuncSetAttribute(k_grid<CfgF64>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)mx);
 }
 
 cudaError_t launch_grid(Prec p, const GridArgs& a, int threads, size_t smem, cudaStream_t s) {
     const int64_t nblocks = (int64_t)a.m_count * a.K * a.r_blocks;
     if (nblocks <= 0 || nblocks > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
-    if (p == Prec::F32) k_grid<Prec::F32><<<(unsigned)nblocks, threads, smem, s>>>(a);
-    else k_grid<Prec::F64><<<(unsigned)nblocks, threads, smem, s>>>(a);
+    if (p == Prec::F32) k_grid<CfgF32><<<(unsigned)nblocks, threads, smem, s>>>(a);
+    else k_grid<CfgF64><<<(unsigned)nblocks, threads, smem, s>>>(a);
     return cudaGetLastError();
 }
 

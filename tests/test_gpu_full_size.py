@@ -1,0 +1,97 @@
+"""CUDA path versus the oracle on the full-size synthetic workloads.
+
+The envelope evaluator of the oracle (the same finite sum regrouped by affine pieces over
+exact cumulative counts, pinned in test_oracle_pins.py) gives every cell of the full grids;
+the direct per-term evaluator checks randomly drawn cells of the same runs.  The 8-class
+workload runs exactly as bench.py times it (FP32, all outputs), plus an FP64 slice.
+"""
+
+import numpy as np
+import pytest
+
+from oracle import oracle as O
+from synth import (drift_loop_workload_k32_n1e6, heavy_tail_workload_k16_n1e6, lognormal_workload_k8_n1e5,
+                   regime_sweep_workload_k8_n2e5, slice_workload)
+from tests.parity import RTOL, compare_full, oracle_from_S, rel_close
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+from paper_2607_16892_gb300 import kvdro  # noqa: E402
+from paper_2607_16892_gb300.runner import run  # noqa: E402
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _need_gpu():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+
+
+def direct_cells(w, gpu_S, n, rtol, seed):
+    """The direct per-term oracle on n random cells (plus each class's first and last r)."""
+    rng = np.random.default_rng(seed)
+    M, K, R, NL = gpu_S.shape
+    m = rng.integers(0, M, n)
+    k = rng.integers(0, K, n)
+    r = rng.integers(0, R, n)
+    l = rng.integers(0, NL, n)
+    m = np.concatenate([m, np.zeros(2 * K, np.int64)])
+    k = np.concatenate([k, np.repeat(np.arange(K), 2)])
+    r = np.concatenate([r, np.tile([0, R - 1], K)])
+    l = np.concatenate([l, rng.integers(0, NL, 2 * K)])
+    ref = O.eval_cells(w, m, k, r, l)
+    return rel_close(gpu_S[m, k, r, l], ref, rtol, "S (direct cells)")
+
+
+def test_lognormal_k8_n1e5_fp32_full_grid_as_benchmarked():
+    w = lognormal_workload_k8_n1e5()
+    gpu = run(w, kvdro.KVDRO_FP32)
+    S_env = O.envelope_grid(w)
+    rep = compare_full(w, gpu, oracle_from_S(w, S_env), "fp32")
+    rep["direct"] = direct_cells(w, gpu["S"], 2048, RTOL["fp32"], 1)
+    assert rep["r_idx_exact"] > 0
+    print(rep)
+
+
+def test_lognormal_k8_n1e5_fp64_slice():
+    w = slice_workload(lognormal_workload_k8_n1e5(), r_index=np.arange(3, 4096, 16), name="k8_fp64_slice")
+    gpu = run(w, kvdro.KVDRO_FP64)
+    compare_full(w, gpu, oracle_from_S(w, O.envelope_grid(w)), "fp64")
+    direct_cells(w, gpu["S"], 1024, RTOL["fp64"], 2)
+
+
+def test_heavy_tail_k16_n1e6_fp32_full_grid():
+    w = heavy_tail_workload_k16_n1e6()
+    gpu = run(w, kvdro.KVDRO_FP32)
+    rep = compare_full(w, gpu, oracle_from_S(w, O.envelope_grid(w)), "fp32")
+    rep["direct"] = direct_cells(w, gpu["S"], 256, RTOL["fp32"], 3)
+    print(rep)
+
+
+def test_regime_sweep_slice_and_critical_fractile():
+    full = regime_sweep_workload_k8_n2e5()
+    mi = np.arange(0, 1024, 16)  # 64 strided regimes, rho from 1 to ~900
+    w = slice_workload(full, regimes=mi, name="regimes_slice")
+    w.fractiles = (w.cp / (w.cp + w.cw)).copy()
+    gpu = run(w, kvdro.KVDRO_FP32)
+    ora = oracle_from_S(w, O.envelope_grid(w))
+    compare_full(w, gpu, ora, "fp32")
+    direct_cells(w, gpu["S"], 256, RTOL["fp32"], 4)
+    # eps = 0 (index 0): the chosen r is the grid point at or just above each regime's critical-fractile
+    # quantile whenever the grid resolves it (Prop. "Critical Fractile Structure").
+    q = O.quantiles(w, w.cp / (w.cp + w.cw))  # [k, m]
+    for mm in range(len(w.cp)):
+        for k in range(w.K):
+            rstar = w.r[gpu["r_idx"][mm, 0, k]]
+            lo = w.r[np.searchsorted(w.r, q[k, mm], side="right") - 1] if q[k, mm] >= w.r[0] else w.r[0]
+            hi = w.r[min(np.searchsorted(w.r, q[k, mm], side="left"), len(w.r) - 1)]
+            assert lo <= rstar <= hi, (mm, k, rstar, q[k, mm])
+
+
+@pytest.mark.parametrize("iteration", [0, 1])
+def test_drift_loop_k32_n1e6_iteration(iteration):
+    w = drift_loop_workload_k32_n1e6(iteration)
+    gpu = run(w, kvdro.KVDRO_FP32)
+    rep = compare_full(w, gpu, oracle_from_S(w, O.envelope_grid(w)), "fp32")
+    rep["direct"] = direct_cells(w, gpu["S"], 128, RTOL["fp32"], 5 + iteration)
+    print(rep)
