@@ -39,9 +39,12 @@ from synth import lognormal_workload_k8_n1e5, slice_workload  # noqa: E402
 METRIC = "DRO cost terms/sec (class×r×λ×sample) on 1 GB300; % of FP32/HBM roofline"
 UNIT = "terms/s"
 SM_MAX_MHZ_RECIPE = 2070.0
-# Issue bound of the FP32 inner loop: per pair of terms one fma.f32x2, two max.f32 and one
-# add.f32x2 = 4 warp instructions, i.e. 2 issue slots per term; 4 schedulers x 32 lanes per SM.
-TERMS_PER_CLK_PER_SM = 64.0
+# FP32 lane-operation bound of the grid kernel: every term costs three FP32 lane-operations (one
+# fused multiply-add, one max, one add), and an SM dispatches at most 4 schedulers x 32 lanes =
+# 128 FP32 lane-operations per clock (a packed f32x2 instruction occupies two dispatch cycles).
+LANE_OPS_PER_CLK_PER_SM = 128.0
+LANE_OPS_PER_TERM = 3.0
+TERMS_PER_CLK_PER_SM = LANE_OPS_PER_CLK_PER_SM / LANE_OPS_PER_TERM
 GRID_SOURCE = os.path.join(ROOT, "paper_2607_16892_gb300", "csrc", "grid.cu")
 PROFILE = os.path.join(ROOT, "profiles", "k_grid_f32_lognormal_k8_n1e5.md")
 LAUNCHES_PER_STEP = 6  # histogram, scan, expand, quantile gather, grid, argmin finalise
@@ -274,8 +277,8 @@ def run_ours(args):
     roofline = {"bound": "alu", "achieved": achieved, "peak": peak, "unit": UNIT, "frac": achieved / peak,
                 "traffic": profile_traffic(), "kernel": "k_grid<F32>",
                 "kernel_ms_mean": kernel_ms,
-                "peak_basis": f"{props.multi_processor_count} SMs x {TERMS_PER_CLK_PER_SM:.0f} terms/clk/SM x "
-                              f"{SM_MAX_MHZ_RECIPE:.0f} MHz (issue bound of the f32x2 inner loop)"}
+                "peak_basis": f"{props.multi_processor_count} SMs x {LANE_OPS_PER_CLK_PER_SM:.0f} FP32 lane-ops/clk/SM "
+                              f"/ {LANE_OPS_PER_TERM:.0f} lane-ops per term x {SM_MAX_MHZ_RECIPE:.0f} MHz"}
     if clocks.get("sm_mhz"):
         roofline["frac_at_sampled_clock"] = achieved / (peak * clocks["sm_mhz"] / SM_MAX_MHZ_RECIPE)
 

@@ -33,7 +33,6 @@ constexpr int32_t kMaxF = 65536;
 constexpr int64_t kMaxKF = 1 << 22;
 constexpr int32_t kMaxNLf32 = 256;
 constexpr int32_t kMaxNLf64 = 128;
-constexpr int kWarpsPerCta = 8;
 
 struct Buf {
     void* p = nullptr;
@@ -431,14 +430,8 @@ int kvdro_eval_grid(kvdro_ctx* ctx, int precision, int32_t R, const int32_t* r, 
     if (!g.ok) return fail(ctx, KVDRO_ECUDA, "cannot select device %d", ctx->device);
     ctx->last_stream = s;
 
-    // Launch shape: LT lam tiles x RG r groups of warps per CTA.
-    const int TL = kvdro::grid_tile_lam(P), TR = kvdro::grid_tile_r(P);
-    const int LT = (NL + TL - 1) / TL;
-    const int RG = LT >= kWarpsPerCta ? 1 : kWarpsPerCta / LT;
-    const int threads = 32 * LT * RG;
-    const int r_per_cta = RG * TR;
-    const int r_blocks = (R + r_per_cta - 1) / r_per_cta;
-    const size_t smem = kvdro::grid_smem_bytes(P, RG, LT, E, NL);
+    // Launch shape: lam tiles x r groups of warps per CTA.
+    const kvdro::GridShape shape = kvdro::grid_shape(P, R, NL, E);
 
     // Grid parameters in one upload.
     const size_t gbytes = align_up((size_t)R * 4, 8) + 8 * ((size_t)NL + E + 2 * (size_t)M);
@@ -520,22 +513,19 @@ int kvdro_eval_grid(kvdro_ctx* ctx, int precision, int32_t R, const int32_t* r, 
     a.NL = NL;
     a.E = E;
     a.M = M;
-    a.LT = LT;
-    a.RG = RG;
-    a.r_blocks = r_blocks;
     a.S_out = outs[0].dev;
     a.cost_out = cost_dev;
     a.lam_idx_out = static_cast<int32_t*>(outs[2].dev);
     a.keys = static_cast<unsigned long long*>(ctx->keys.p);
     a.err = static_cast<int32_t*>(ctx->errs.p);
-    const int64_t per_m = (int64_t)ctx->K * r_blocks;
+    const int64_t per_m = (int64_t)ctx->K * shape.r_blocks;
     const int64_t m_step = std::max<int64_t>(1, 0x7fffffffLL / per_m);
     ctx->grid_timed = false;
     KV_CUDA(cudaEventRecord(ctx->grid_t0, s), "recording grid start");
     for (int64_t m0 = 0; m0 < M; m0 += m_step) {
         a.m0 = (int32_t)m0;
         a.m_count = (int32_t)std::min<int64_t>(m_step, M - m0);
-        KV_CUDA(kvdro::launch_grid(P, a, threads, smem, s), "grid kernel");
+        KV_CUDA(kvdro::launch_grid(P, shape, a, s), "grid kernel");
     }
     KV_CUDA(cudaEventRecord(ctx->grid_t1, s), "recording grid end");
     ctx->grid_timed = true;

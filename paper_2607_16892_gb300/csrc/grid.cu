@@ -42,16 +42,22 @@ constexpr int ilog2(int v) { return v <= 1 ? 0 : 1 + ilog2(v / 2); }
 
 // Shape of one instantiation of the grid kernel: precision, warp tile (TR reservations x TL
 // multipliers, TR*TL a power of two <= 32), FP32 chunks between folds of the per-lane partial
-// sums into FP64 (FP64 folds once at the end), and the minimum CTAs per SM it is built for.
-template <Prec P_, int TR_, int TL_, int FLUSH_, int MINB_>
+// sums into FP64 (FP64 folds once at the end), and the largest CTA and minimum CTAs per SM it is
+// compiled for (these two bound its registers per thread).
+template <Prec P_, int TR_, int TL_, int FLUSH_, int MINB_, int MAXT_ = 512>
 struct GridCfg {
     static constexpr Prec P = P_;
     static constexpr int TR = TR_, TL = TL_, V = TR_ * TL_, LOG2V = ilog2(TR_ * TL_), FLUSH = FLUSH_, MINB = MINB_;
+    static constexpr int MAXT = MAXT_;
     static_assert((V & (V - 1)) == 0 && V >= 2 && V <= 32, "tile must hold a power of two <= 32 cells");
     static_assert(P_ == Prec::F64 || TL_ % 2 == 0, "the FP32 tile packs lam values in pairs");
 };
-using CfgF32 = GridCfg<Prec::F32, 2, 16, 2, 1>;
-using CfgF64 = GridCfg<Prec::F64, 2, 8, 0, 1>;
+// FP32: 2 r x 8 lam tiles, up to 16 warps per CTA and two CTAs per SM (64 registers) for up to
+// 128 lam values; 2 x 16 tiles for 129..256 lam values.  FP64: 2 x 8 tiles.
+using CfgF32 = GridCfg<Prec::F32, 2, 8, 4, 2, 512>;
+using CfgF32Wide = GridCfg<Prec::F32, 2, 16, 4, 1, 512>;
+using CfgF64 = GridCfg<Prec::F64, 2, 8, 0, 1, 512>;
+constexpr int kWarpsTarget = 16;  // warps per CTA the r groups fill up to
 
 // ---------------------------------------------------------------- PTX helpers
 
@@ -170,7 +176,7 @@ __host__ __device__ inline SmemLayout smem_layout(int RG, int TR, int NLpad, int
 // ---------------------------------------------------------------- the grid kernel
 
 template <class C>
-__global__ void __launch_bounds__(kMaxThreads, C::MINB) k_grid(const GridArgs a) {
+__global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
     constexpr Prec P = C::P;
     constexpr int TR = C::TR, TL = C::TL, V = C::V, LOG2V = C::LOG2V;
     extern __shared__ __align__(128) unsigned char smem[];
@@ -257,21 +263,16 @@ __global__ void __launch_bounds__(kMaxThreads, C::MINB) k_grid(const GridArgs a)
                 for (int t = 0; t < nq; t++) {
                     const float4 v = q[lane + 32 * t];
                     const u64 xa = pk(v.x, v.y), xb = pk(v.z, v.w);
+                    // The two samples' excesses are added to each other before they join the running
+                    // sum: the same number of adds, half as many additions into the long sum.
 #pragma unroll
                     for (int i = 0; i < TR; i++)
 #pragma unroll
                         for (int jp = 0; jp < TL / 2; jp++) {
-                            float w0, w1;
-                            upk(ffma2(kap[jp], xa, dd[i][jp]), w0, w1);
-                            acc[i][jp] = fadd2(acc[i][jp], pk(relu(w0), relu(w1)));
-                        }
-#pragma unroll
-                    for (int i = 0; i < TR; i++)
-#pragma unroll
-                        for (int jp = 0; jp < TL / 2; jp++) {
-                            float w0, w1;
-                            upk(ffma2(kap[jp], xb, dd[i][jp]), w0, w1);
-                            acc[i][jp] = fadd2(acc[i][jp], pk(relu(w0), relu(w1)));
+                            float a0, a1, b0, b1;
+                            upk(ffma2(kap[jp], xa, dd[i][jp]), a0, a1);
+                            upk(ffma2(kap[jp], xb, dd[i][jp]), b0, b1);
+                            acc[i][jp] = fadd2(acc[i][jp], fadd2(pk(relu(a0), relu(a1)), pk(relu(b0), relu(b1))));
                         }
                 }
                 // Every C::FLUSH chunks (and after the last), fold the FP32 partials into the FP64
@@ -455,26 +456,42 @@ __global__ void k_finalize(const FinalizeArgs a) {
 
 }  // namespace
 
-int grid_tile_r(Prec p) { return p == Prec::F32 ? CfgF32::TR : CfgF64::TR; }
-int grid_tile_lam(Prec p) { return p == Prec::F32 ? CfgF32::TL : CfgF64::TL; }
+template <class C>
+GridShape shape_for(int variant, int32_t R, int32_t NL, int32_t E) {
+    GridShape sh;
+    sh.variant = variant;
+    sh.LT = (NL + C::TL - 1) / C::TL;
+    sh.RG = sh.LT >= kWarpsTarget ? 1 : kWarpsTarget / sh.LT;
+    sh.threads = 32 * sh.LT * sh.RG;
+    sh.r_blocks = (R + sh.RG * C::TR - 1) / (sh.RG * C::TR);
+    sh.smem = smem_layout(sh.RG, C::TR, sh.LT * C::TL, E).total;
+    return sh;
+}
 
-size_t grid_smem_bytes(Prec p, int RG, int LT, int E, int NL) {
-    (void)NL;
-    return smem_layout(RG, grid_tile_r(p), LT * grid_tile_lam(p), E).total;
+GridShape grid_shape(Prec p, int32_t R, int32_t NL, int32_t E) {
+    if (p == Prec::F64) return shape_for<CfgF64>(2, R, NL, E);
+    if (NL <= kWarpsTarget * CfgF32::TL) return shape_for<CfgF32>(0, R, NL, E);
+    return shape_for<CfgF32Wide>(1, R, NL, E);
 }
 
 cudaError_t grid_prepare(Prec p) {
-    // the largest layout: 16 warps, 256 lam, 64 eps
-    const size_t mx = smem_layout(8, 2, 256, 64).total + 4096;
-    if (p == Prec::F32) return cudaFuncSetAttribute(k_grid<CfgF32>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)mx);
-    return cudaFuncSetAttribute(k_grid<CfgF64>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)mx);
+    // the largest layout any variant can need: 16 warps, 256 lam, 64 eps
+    const int mx = (int)(smem_layout(16, 2, 256, 64).total + 4096);
+    if (p == Prec::F64) return cudaFuncSetAttribute(k_grid<CfgF64>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
+    cudaError_t e = cudaFuncSetAttribute(k_grid<CfgF32>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
+    if (e != cudaSuccess) return e;
+    return cudaFuncSetAttribute(k_grid<CfgF32Wide>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
 }
 
-cudaError_t launch_grid(Prec p, const GridArgs& a, int threads, size_t smem, cudaStream_t s) {
+cudaError_t launch_grid(Prec p, const GridShape& sh, GridArgs a, cudaStream_t s) {
+    a.LT = sh.LT;
+    a.RG = sh.RG;
+    a.r_blocks = sh.r_blocks;
     const int64_t nblocks = (int64_t)a.m_count * a.K * a.r_blocks;
     if (nblocks <= 0 || nblocks > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
-    if (p == Prec::F32) k_grid<CfgF32><<<(unsigned)nblocks, threads, smem, s>>>(a);
-    else k_grid<CfgF64><<<(unsigned)nblocks, threads, smem, s>>>(a);
+    if (p == Prec::F64) k_grid<CfgF64><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
+    else if (sh.variant == 0) k_grid<CfgF32><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
+    else k_grid<CfgF32Wide><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
     return cudaGetLastError();
 }
 

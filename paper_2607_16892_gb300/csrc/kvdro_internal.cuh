@@ -81,11 +81,19 @@ struct FinalizeArgs {
 };
 
 // grid.cu
-int grid_tile_r(Prec p);                      // r values per warp tile
-int grid_tile_lam(Prec p);                    // lam values per warp tile
-size_t grid_smem_bytes(Prec p, int RG, int LT, int E, int NL);
-cudaError_t grid_prepare(Prec p);             // one-time per-device attribute setup
-cudaError_t launch_grid(Prec p, const GridArgs& a, int threads, size_t smem, cudaStream_t s);
+// Launch shape of the grid kernel for one (precision, grid) problem: which compiled variant,
+// lam tiles x r groups of warps per CTA, CTAs per (regime, class), dynamic shared memory.
+struct GridShape {
+    int variant;       // index of the compiled kernel instantiation
+    int LT, RG;        // lam tiles and r groups per CTA
+    int threads;       // 32 * LT * RG
+    int r_blocks;      // CTAs per (m, k)
+    size_t smem;
+};
+GridShape grid_shape(Prec p, int32_t R, int32_t NL, int32_t E);
+cudaError_t grid_prepare(Prec p);             // per-device attribute setup of every variant of p
+// Launches over regimes [a.m0, a.m0 + a.m_count); fills a.LT, a.RG, a.r_blocks from `sh`.
+cudaError_t launch_grid(Prec p, const GridShape& sh, GridArgs a, cudaStream_t s);
 cudaError_t launch_finalize(Prec p, const FinalizeArgs& a, cudaStream_t s);
 
 }  // namespace kvdro

@@ -248,10 +248,7 @@ extern "C" int kvdro_eval_grid_noalloc(int32_t K, const int64_t* offsets, const 
     if (bad) return report(err, err_len, KVDRO_EINVAL, "samples outside [0, L_max] of their class");
 
     // ---- the FP32 grid kernel and the argmin finalisation
-    const int TL = kvdro::grid_tile_lam(kvdro::Prec::F32), TR = kvdro::grid_tile_r(kvdro::Prec::F32);
-    const int LT = (NL + TL - 1) / TL;
-    const int RG = LT >= 8 ? 1 : 8 / LT;
-    const int r_blocks = (R + RG * TR - 1) / (RG * TR);
+    const kvdro::GridShape shape = kvdro::grid_shape(kvdro::Prec::F32, R, NL, E);
     kvdro::GridArgs a;
     a.pairs = sa.pairs;
     a.pair_off = sa.pair_off;
@@ -271,21 +268,17 @@ extern "C" int kvdro_eval_grid_noalloc(int32_t K, const int64_t* offsets, const 
     a.NL = NL;
     a.E = E;
     a.M = M;
-    a.LT = LT;
-    a.RG = RG;
-    a.r_blocks = r_blocks;
     a.S_out = nullptr;
     a.cost_out = cost;
     a.lam_idx_out = lam_idx;
     a.keys = reinterpret_cast<unsigned long long*>(S + o_keys);
     a.err = sa.err;
-    const int64_t per_m = (int64_t)K * r_blocks;
+    const int64_t per_m = (int64_t)K * shape.r_blocks;
     const int64_t m_step = per_m > 0x7fffffffLL ? 1 : 0x7fffffffLL / per_m;
     for (int64_t m0 = 0; m0 < M; m0 += m_step) {
         a.m0 = (int32_t)m0;
         a.m_count = (int32_t)(m_step < M - m0 ? m_step : M - m0);
-        NA_CUDA(kvdro::launch_grid(kvdro::Prec::F32, a, 32 * LT * RG,
-                                   kvdro::grid_smem_bytes(kvdro::Prec::F32, RG, LT, E, NL), s));
+        NA_CUDA(kvdro::launch_grid(kvdro::Prec::F32, shape, a, s));
     }
     kvdro::FinalizeArgs fa;
     fa.keys = a.keys;

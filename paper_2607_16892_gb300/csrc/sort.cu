@@ -140,7 +140,21 @@ __global__ void __launch_bounds__(kExpandThreads) k_expand(SortArgs a) {
         for (int j = 0; j < kExpandPerThread; j++) {
             const int64_t p = p0 + j;
             if (p < Nk) {
-                while (v < Lk && (int64_t)__ldg(C + v) <= p) v++;  // bounded even if samples were rejected
+                if ((int64_t)__ldg(C + v) <= p) {
+                    // Galloping search for the next bin: doubling steps, then bisection.  Gaps between
+                    // consecutive sorted values can span thousands of empty bins in a heavy tail.
+                    int32_t base = v, step = 1;  // invariant: C[base] <= p
+                    while (step <= Lk - base && (int64_t)__ldg(C + base + step) <= p) {
+                        base += step;
+                        step <<= 1;
+                    }
+                    int32_t a = min(base + 1, Lk), b2 = (step <= Lk - base) ? base + step : Lk;  // both <= Lk
+                    while (a < b2) {
+                        const int32_t mid = (a + b2) >> 1;
+                        if ((int64_t)__ldg(C + mid) > p) b2 = mid; else a = mid + 1;
+                    }
+                    v = a;
+                }
                 out[p] = v;
                 vals[j] = (float)v;
             } else {
