@@ -55,7 +55,10 @@ typedef enum {
 
 typedef enum {
     KVDRO_FP32 = 0,      /* per-term arithmetic in FP32; sums folded into FP64 */
-    KVDRO_FP64 = 1       /* per-term arithmetic and sums in FP64 */
+    KVDRO_FP64 = 1,      /* per-term arithmetic and sums in FP64 */
+    KVDRO_EXACT = 2      /* per-term FP32 decisions on exact integer thresholds, exact integer
+                            counts and sample sums, combined once per cell in FP64; results
+                            carry FP64 rounding only.  Needs every L_max <= 2^22. */
 } kvdro_precision;
 
 /* Create a context on CUDA device `device_ordinal`.  *out receives the handle (NULL on error). */
@@ -87,10 +90,10 @@ int kvdro_quantiles(kvdro_ctx* ctx, int32_t F, const double* fractiles, int32_t*
 
 /*
  * Evaluate the grid and reduce it.  Element type of S, cost and min_cost is float for
- * KVDRO_FP32 and double for KVDRO_FP64.
+ * KVDRO_FP32 and double for KVDRO_FP64 and KVDRO_EXACT.
  *   R, r       host int32[R], 1 <= R <= 2^20; every r must satisfy L_in_k <= r <= L_in_k + L_k for
  *              every class (the reservation domain of Sec. 2.2).
- *   NL, lam    host double[NL], finite, >= 0; 1 <= NL <= 256 (FP32) or 128 (FP64).
+ *   NL, lam    host double[NL], finite, >= 0; 1 <= NL <= 256 (FP32) or 128 (FP64, EXACT).
  *   E, eps     host double[E], finite, >= 0; 1 <= E <= 64.
  *   M, c_p,c_w host double[M] each, finite, >= 0; 1 <= M <= 65536.
  * Outputs (each may be NULL to skip it; host or device):

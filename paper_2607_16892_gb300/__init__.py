@@ -7,6 +7,7 @@ The computation lives in the CUDA library built from ``csrc/`` (C ABI in
 from . import kvdro  # noqa: F401
 from .kvdro import (  # noqa: F401
     KVDRO_FP32,
+    KVDRO_EXACT,
     KVDRO_FP64,
     KvdroError,
     kvdro_create,

@@ -208,7 +208,8 @@ int kvdro_create(kvdro_ctx** out, int device_ordinal) {
     DeviceGuard g(device_ordinal);
     if (!g.ok || kvdro::grid_prepare(Prec::F32) != cudaSuccess || kvdro::grid_prepare(Prec::F64) != cudaSuccess ||
         cudaEventCreateWithFlags(&ctx->pin_free, cudaEventDisableTiming) != cudaSuccess ||
-        cudaEventCreate(&ctx->grid_t0) != cudaSuccess || cudaEventCreate(&ctx->grid_t1) != cudaSuccess) {
+        kvdro::grid_prepare(Prec::EXACT) != cudaSuccess || cudaEventCreate(&ctx->grid_t0) != cudaSuccess ||
+        cudaEventCreate(&ctx->grid_t1) != cudaSuccess) {
         cudaGetLastError();
         delete ctx;
         return KVDRO_ECUDA;
@@ -406,10 +407,14 @@ int kvdro_eval_grid(kvdro_ctx* ctx, int precision, int32_t R, const int32_t* r, 
     if (!ctx) return KVDRO_EINVAL;
     ctx->err.clear();
     if (!ctx->loaded) return fail(ctx, KVDRO_ESTATE, "no samples loaded");
-    if (precision != KVDRO_FP32 && precision != KVDRO_FP64)
-        return fail(ctx, KVDRO_EINVAL, "precision must be KVDRO_FP32 or KVDRO_FP64");
-    const Prec P = precision == KVDRO_FP32 ? Prec::F32 : Prec::F64;
+    if (precision != KVDRO_FP32 && precision != KVDRO_FP64 && precision != KVDRO_EXACT)
+        return fail(ctx, KVDRO_EINVAL, "precision must be KVDRO_FP32, KVDRO_FP64 or KVDRO_EXACT");
+    const Prec P = precision == KVDRO_FP32 ? Prec::F32 : precision == KVDRO_FP64 ? Prec::F64 : Prec::EXACT;
     const int32_t maxNL = P == Prec::F32 ? kMaxNLf32 : kMaxNLf64;
+    if (P == Prec::EXACT)
+        for (int32_t k = 0; k < ctx->K; k++)
+            if (ctx->L[k] > kvdro::kExactMaxL)
+                return fail(ctx, KVDRO_EINVAL, "KVDRO_EXACT needs L_max <= 2^22 (class %d has %d)", k, ctx->L[k]);
     if (R < 1 || R > kMaxR) return fail(ctx, KVDRO_EINVAL, "R = %d outside [1, 2^20]", R);
     if (NL < 1 || NL > maxNL) return fail(ctx, KVDRO_EINVAL, "NL = %d outside [1, %d]", NL, maxNL);
     if (E < 1 || E > kMaxE) return fail(ctx, KVDRO_EINVAL, "E = %d outside [1, %d]", E, kMaxE);
@@ -487,7 +492,7 @@ int kvdro_eval_grid(kvdro_ctx* ctx, int precision, int32_t R, const int32_t* r, 
             }
     }
     void* cost_dev = outs[1].dev;
-    if (P == Prec::F64 && !cost_dev) {  // FP64 min_cost is read back from the cost array
+    if (P != Prec::F32 && !cost_dev) {  // FP64 / EXACT min_cost is read back from the cost array
         if ((rc = ensure(ctx, ctx->cost64, (size_t)cells_out * 8))) return rc;
         cost_dev = ctx->cost64.p;
     }

@@ -35,7 +35,6 @@ typedef unsigned long long u64;
 
 constexpr int kChunk = 2048;      // samples per staged chunk (16 KB of float2)
 constexpr int kStages = 3;        // ring depth
-constexpr int kMaxThreads = 512;  // up to 16 warps per CTA
 constexpr long long kWaitCycles = 4000000000LL;  // ~2 s at 2 GHz: bound on any barrier wait
 
 constexpr int ilog2(int v) { return v <= 1 ? 0 : 1 + ilog2(v / 2); }
@@ -50,13 +49,14 @@ struct GridCfg {
     static constexpr int TR = TR_, TL = TL_, V = TR_ * TL_, LOG2V = ilog2(TR_ * TL_), FLUSH = FLUSH_, MINB = MINB_;
     static constexpr int MAXT = MAXT_;
     static_assert((V & (V - 1)) == 0 && V >= 2 && V <= 32, "tile must hold a power of two <= 32 cells");
-    static_assert(P_ == Prec::F64 || TL_ % 2 == 0, "the FP32 tile packs lam values in pairs");
+    static_assert(P_ == Prec::F64 || TL_ % 2 == 0, "the FP32 and exact tiles pack lam values in pairs");
 };
 // FP32: 2 r x 8 lam tiles, up to 16 warps per CTA and two CTAs per SM (64 registers) for up to
 // 128 lam values; 2 x 16 tiles for 129..256 lam values.  FP64: 2 x 8 tiles.
 using CfgF32 = GridCfg<Prec::F32, 2, 8, 4, 2, 512>;
 using CfgF32Wide = GridCfg<Prec::F32, 2, 16, 4, 1, 512>;
 using CfgF64 = GridCfg<Prec::F64, 2, 8, 0, 1, 512>;
+using CfgExact = GridCfg<Prec::EXACT, 2, 8, 0, 2, 512>;
 constexpr int kWarpsTarget = 16;  // warps per CTA the r groups fill up to
 
 // ---------------------------------------------------------------- PTX helpers
@@ -89,6 +89,32 @@ __device__ __forceinline__ double relu(double w) {
     double d;
     asm("max.f64 %0, %1, 0d0000000000000000;" : "=d"(d) : "d"(w));
     return d;
+}
+
+// min(max(a + b, 0), 1) in one FMA-pipe instruction.  With a an integer sample and b = 1 - t for
+// an integer threshold t this is exactly the indicator [a >= t]: a + 1 - t is an integer, >= 1
+// when a >= t and <= 0 otherwise, and rounding cannot move an integer across that gap.
+__device__ __forceinline__ float sat_add(float a, float b) {
+    float d;
+    asm("add.rn.sat.f32 %0, %1, %2;" : "=f"(d) : "f"(a), "f"(b));
+    return d;
+}
+// max(x, -2): padding samples (NaN) become -2, below every threshold; real samples (>= 0) pass.
+__device__ __forceinline__ float clamp_pad(float x) {
+    float d;
+    asm("max.f32 %0, %1, 0fC0000000;" : "=f"(d) : "f"(x));
+    return d;
+}
+
+// Smallest integer t with kappa * t + d > 0, clamped to [-1, 2^23] (so 1 - t is exact in FP32).
+// For integer samples x <= 2^22, x >= t exactly when max(kappa x + d, 0) is positive; a sample
+// at the boundary has kappa x + d within a rounding of zero, so either choice adds nothing
+// material.  2^23 means "never active".
+__device__ __forceinline__ float exact_threshold(double kappa, double d) {
+    if (!(kappa > 0.0)) return d > 0.0 ? -1.0f : 8388608.0f;
+    double t = floor(-d / kappa) + 1.0;
+    t = fmin(fmax(t, -1.0), 8388608.0);
+    return (float)t;
 }
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
@@ -302,7 +328,7 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
                 issued = c + kStages + 1;
             }
         }
-    } else {
+    } else if constexpr (P == Prec::F64) {
         double kap[TL], dd[TR][TL], acc[TR][TL];
 #pragma unroll
         for (int j = 0; j < TL; j++) {
@@ -357,6 +383,109 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
                 for (int j = 0; j < TL; j++) vals[i * TL + j] = acc[i][j];
             acc64 = transpose_reduce<double, V>(vals, lane);
         }
+    } else {
+        // EXACT: per cell (i, j), the active samples are those with x >= t_ij; the kernel counts them
+        // and sums them exactly (FP32 holds every integer below 2^24), and the epilogue forms
+        // kappa * sum + d * count in FP64.
+        u64 nt[TR][TL / 2], sx[TR][TL / 2], cn[TR][TL / 2];  // nt holds 1 - t per cell
+#pragma unroll
+        for (int jp = 0; jp < TL / 2; jp++) {
+            const int j0 = lt * TL + 2 * jp;
+            const double l0 = s_lam[j0], l1 = s_lam[j0 + 1];
+            const bool v0 = j0 < a.NL, v1 = j0 + 1 < a.NL;
+            const double mu0 = fmin(l0, cp), mu1 = fmin(l1, cp);
+            const double k0 = mu0 + fmin(l0, cw), k1 = mu1 + fmin(l1, cw);
+#pragma unroll
+            for (int i = 0; i < TR; i++) {
+                const float t0 = (v0 && rvalid[i]) ? exact_threshold(k0, (cp - mu0) * Lk - (cp + cw) * eta[i]) : 8388608.0f;
+                const float t1 = (v1 && rvalid[i]) ? exact_threshold(k1, (cp - mu1) * Lk - (cp + cw) * eta[i]) : 8388608.0f;
+                nt[i][jp] = pk(1.0f - t0, 1.0f - t1);
+                sx[i][jp] = 0ull;
+                cn[i][jp] = 0ull;
+            }
+        }
+        // Fold the FP32 sums into int64 after `fe` loads of two samples: per-lane sums stay below
+        // 2 * fe * L <= 2^23 (fe is a power of two, the same for every thread of the CTA).
+        int fe = 1;
+        while (fe < 1024 && 2 * (int64_t)(2 * fe) * a.L[k] <= (1ll << 23)) fe <<= 1;
+        long long acc_sx = 0, acc_cn = 0;
+        auto fold = [&]() {
+            int vs[V], vc[V];
+#pragma unroll
+            for (int i = 0; i < TR; i++)
+#pragma unroll
+                for (int jp = 0; jp < TL / 2; jp++) {
+                    float a0, a1, b0, b1;
+                    upk(sx[i][jp], a0, a1);
+                    upk(cn[i][jp], b0, b1);
+                    vs[i * TL + 2 * jp] = __float2int_rn(a0);
+                    vs[i * TL + 2 * jp + 1] = __float2int_rn(a1);
+                    vc[i * TL + 2 * jp] = __float2int_rn(b0);
+                    vc[i * TL + 2 * jp + 1] = __float2int_rn(b1);
+                    sx[i][jp] = 0ull;
+                    cn[i][jp] = 0ull;
+                }
+            acc_sx += (long long)transpose_reduce<int, V>(vs, lane);
+            acc_cn += (long long)transpose_reduce<int, V>(vc, lane);
+        };
+        int pending = 0;  // loads since the last fold
+        for (int c = 0; c < nchunks; c++) {
+            const int s = c % kStages;
+            if (!mbar_wait_bounded(smem_u32(&full[s]), (uint32_t)((c / kStages) & 1))) timeout = true;
+            if (!timeout) {
+                const int cnt = (int)min((int64_t)kChunk, np - (int64_t)c * kChunk);
+                const float4* q = reinterpret_cast<const float4*>(ring + (size_t)s * kChunk);
+                const int nq = cnt >> 6;
+                for (int t0 = 0; t0 < nq; t0 += fe) {
+                    const int t1 = min(nq, t0 + fe);
+                    for (int t = t0; t < t1; t++) {
+                        const float4 v = q[lane + 32 * t];
+                        const float xa0 = clamp_pad(v.x), xa1 = clamp_pad(v.y);
+                        const float xb0 = clamp_pad(v.z), xb1 = clamp_pad(v.w);
+                        const u64 xa = pk(xa0, xa1), xb = pk(xb0, xb1);
+#pragma unroll
+                        for (int i = 0; i < TR; i++)
+#pragma unroll
+                            for (int jp = 0; jp < TL / 2; jp++) {
+                                float n0, n1;
+                                upk(nt[i][jp], n0, n1);
+                                const u64 pa = pk(sat_add(xa0, n0), sat_add(xa1, n1));
+                                const u64 pb = pk(sat_add(xb0, n0), sat_add(xb1, n1));
+                                sx[i][jp] = ffma2(pb, xb, ffma2(pa, xa, sx[i][jp]));
+                                cn[i][jp] = fadd2(cn[i][jp], fadd2(pa, pb));
+                            }
+                    }
+                    pending += t1 - t0;
+                    if (pending >= fe) {
+                        fold();
+                        pending = 0;
+                    }
+                }
+            }
+            consumed = c;
+            if (__syncthreads_or(timeout)) {
+                timeout = true;
+                break;
+            }
+            if (c + kStages < nchunks) {
+                if (tid == 0) {
+                    fence_proxy_async();
+                    issue(c + kStages);
+                }
+                issued = c + kStages + 1;
+            }
+        }
+        if (!timeout) {
+            if (pending > 0) fold();
+            // this lane's cell: kappa * sum + d * count in FP64
+            const int cidx = lane >> (5 - LOG2V);
+            const int i = cidx / TL, j = cidx % TL;
+            const int lj = lt * TL + j;
+            const double l = lj < a.NL ? s_lam[lj] : 0.0;
+            const double mu = fmin(l, cp), kap = mu + fmin(l, cw);
+            const double d = (cp - mu) * Lk - (cp + cw) * eta[i];
+            acc64 = kap * (double)acc_sx + d * (double)acc_cn;
+        }
     }
 
     if (timeout) {
@@ -386,7 +515,7 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
             if (a.S_out) {
                 const size_t o = (((size_t)m * a.K + k) * a.R + ri) * a.NL + lj;
                 if constexpr (P == Prec::F32) static_cast<float*>(a.S_out)[o] = (float)S;
-                else static_cast<double*>(a.S_out)[o] = S;
+                else static_cast<double*>(a.S_out)[o] = S;  // F64 and EXACT
             }
         }
     }
@@ -470,6 +599,7 @@ GridShape shape_for(int variant, int32_t R, int32_t NL, int32_t E) {
 
 GridShape grid_shape(Prec p, int32_t R, int32_t NL, int32_t E) {
     if (p == Prec::F64) return shape_for<CfgF64>(2, R, NL, E);
+    if (p == Prec::EXACT) return shape_for<CfgExact>(3, R, NL, E);
     if (NL <= kWarpsTarget * CfgF32::TL) return shape_for<CfgF32>(0, R, NL, E);
     return shape_for<CfgF32Wide>(1, R, NL, E);
 }
@@ -478,6 +608,7 @@ cudaError_t grid_prepare(Prec p) {
     // the largest layout any variant can need: 16 warps, 256 lam, 64 eps
     const int mx = (int)(smem_layout(16, 2, 256, 64).total + 4096);
     if (p == Prec::F64) return cudaFuncSetAttribute(k_grid<CfgF64>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
+    if (p == Prec::EXACT) return cudaFuncSetAttribute(k_grid<CfgExact>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
     cudaError_t e = cudaFuncSetAttribute(k_grid<CfgF32>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
     if (e != cudaSuccess) return e;
     return cudaFuncSetAttribute(k_grid<CfgF32Wide>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
@@ -490,6 +621,7 @@ cudaError_t launch_grid(Prec p, const GridShape& sh, GridArgs a, cudaStream_t s)
     const int64_t nblocks = (int64_t)a.m_count * a.K * a.r_blocks;
     if (nblocks <= 0 || nblocks > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
     if (p == Prec::F64) k_grid<CfgF64><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
+    else if (p == Prec::EXACT) k_grid<CfgExact><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
     else if (sh.variant == 0) k_grid<CfgF32><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
     else k_grid<CfgF32Wide><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
     return cudaGetLastError();

@@ -38,7 +38,10 @@ cudaError_t launch_expand(const SortArgs& a, int32_t nblocks, cudaStream_t s);
 cudaError_t launch_gather_quantiles(const int32_t* sorted, const int64_t* offsets, const int32_t* rank, int32_t K,
                                     int32_t F, int32_t* out, cudaStream_t s);
 
-enum class Prec { F32 = 0, F64 = 1 };
+// F32: per-term FP32 excess sums folded into FP64.  F64: per-term FP64.  EXACT: per-term FP32
+// threshold decisions with exact integer count and sample-sum accumulation, combined in FP64.
+enum class Prec { F32 = 0, F64 = 1, EXACT = 2 };
+constexpr int32_t kExactMaxL = 1 << 22;  // EXACT needs 2 * L < 2^23 per fold of two samples
 
 struct GridArgs {
     const float2* pairs;        // padded (x, x) pairs

@@ -31,6 +31,7 @@ KVDRO_ESTATE = -4
 KVDRO_ETIMEOUT = -5
 KVDRO_FP32 = 0
 KVDRO_FP64 = 1
+KVDRO_EXACT = 2
 
 _STATUS = {0: "KVDRO_OK", -1: "KVDRO_EINVAL", -2: "KVDRO_ENOMEM", -3: "KVDRO_ECUDA", -4: "KVDRO_ESTATE",
            -5: "KVDRO_ETIMEOUT"}

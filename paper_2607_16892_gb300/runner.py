@@ -10,7 +10,7 @@ from typing import Dict, Iterable, Optional
 
 import numpy as np
 
-from .kvdro import (KVDRO_FP32, KVDRO_FP64, kvdro_create, kvdro_destroy, kvdro_eval_grid, kvdro_load_samples,
+from .kvdro import (KVDRO_EXACT, KVDRO_FP32, KVDRO_FP64, kvdro_create, kvdro_destroy, kvdro_eval_grid, kvdro_load_samples,
                     kvdro_quantiles, kvdro_sorted_samples)
 
 ALL_OUTPUTS = ("S", "cost", "lam_idx", "r_idx", "min_cost", "fhat", "quant", "sorted")

@@ -12,7 +12,7 @@ from __future__ import annotations
 
 import numpy as np
 
-RTOL = {"fp32": 1e-5, "fp64": 1e-9}
+RTOL = {"fp32": 1e-5, "fp64": 1e-9, "exact": 1e-9}
 
 
 def rel_close(gpu, ref, rtol, what="", floor=0.0):

@@ -53,6 +53,23 @@ def test_lognormal_k8_n1e5_fp32_full_grid_as_benchmarked():
     print(rep)
 
 
+def test_lognormal_k8_n1e5_exact_full_grid():
+    """The exact mode on every cell of the benchmarked grid, at the FP64 tolerance."""
+    w = lognormal_workload_k8_n1e5()
+    gpu = run(w, kvdro.KVDRO_EXACT)
+    rep = compare_full(w, gpu, oracle_from_S(w, O.envelope_grid(w)), "exact")
+    rep["direct"] = direct_cells(w, gpu["S"], 1024, RTOL["exact"], 7)
+    print(rep)
+
+
+def test_heavy_tail_k16_n1e6_exact_full_grid():
+    w = heavy_tail_workload_k16_n1e6()
+    gpu = run(w, kvdro.KVDRO_EXACT)
+    rep = compare_full(w, gpu, oracle_from_S(w, O.envelope_grid(w)), "exact")
+    rep["direct"] = direct_cells(w, gpu["S"], 128, RTOL["exact"], 8)
+    print(rep)
+
+
 def test_lognormal_k8_n1e5_fp64_slice():
     w = slice_workload(lognormal_workload_k8_n1e5(), r_index=np.arange(3, 4096, 16), name="k8_fp64_slice")
     gpu = run(w, kvdro.KVDRO_FP64)

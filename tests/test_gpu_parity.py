@@ -20,7 +20,7 @@ pytestmark = pytest.mark.gpu
 from paper_2607_16892_gb300 import kvdro  # noqa: E402
 from paper_2607_16892_gb300.runner import run  # noqa: E402
 
-P = {"fp32": kvdro.KVDRO_FP32, "fp64": kvdro.KVDRO_FP64}
+P = {"fp32": kvdro.KVDRO_FP32, "fp64": kvdro.KVDRO_FP64, "exact": kvdro.KVDRO_EXACT}
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -42,7 +42,7 @@ def make(samples_per_class, L, r, lam, eps, cp, cw, L_in=None, fractiles=(0.0, 0
                     fractiles=np.asarray(fractiles, np.float64))
 
 
-@pytest.mark.parametrize("prec", ["fp64", "fp32"])
+@pytest.mark.parametrize("prec", ["fp64", "fp32", "exact"])
 @pytest.mark.parametrize("seed", [1, 2, 3])
 def test_random_ragged_cases(prec, seed):
     w = random_case(seed, K=3, N=(5000, 777, 33), L=(3000, 3000, 3000), R=45, n_lam=37, n_eps=4, M=3,
@@ -51,22 +51,22 @@ def test_random_ragged_cases(prec, seed):
     compare_full(w, gpu, O.solve(w), prec)
 
 
-@pytest.mark.parametrize("prec", ["fp64", "fp32"])
+@pytest.mark.parametrize("prec", ["fp64", "fp32", "exact"])
 def test_per_class_support_and_input_length(prec):
     w = random_case(7, K=4, N=(2100, 129, 128, 1), L=(900, 1500, 2000, 1200), L_in=(0, 50, 10, 200), R=33,
                     n_lam=16, n_eps=3, M=2, integer_costs=True)
     compare_full(w, run(w, P[prec]), O.solve(w), prec)
 
 
-@pytest.mark.parametrize("prec", ["fp64", "fp32"])
+@pytest.mark.parametrize("prec", ["fp64", "fp32", "exact"])
 def test_lognormal_k3_n1e3_full_grid(prec):
     w = lognormal_workload_k3_n1e3()
     rep = compare_full(w, run(w, P[prec]), O.solve(w), prec)
-    if prec == "fp64":
+    if prec != "fp32":
         assert rep["r_idx_exact"] > 0
 
 
-@pytest.mark.parametrize("prec", ["fp64", "fp32"])
+@pytest.mark.parametrize("prec", ["fp64", "fp32", "exact"])
 def test_max_lambda_grid_and_single_points(prec):
     nl = 256 if prec == "fp32" else 128
     rng = np.random.default_rng(5)
@@ -77,7 +77,7 @@ def test_max_lambda_grid_and_single_points(prec):
     compare_full(w1, run(w1, P[prec]), O.solve(w1), prec)
 
 
-@pytest.mark.parametrize("prec", ["fp64", "fp32"])
+@pytest.mark.parametrize("prec", ["fp64", "fp32", "exact"])
 def test_degenerate_inputs(prec):
     L = 64
     cases = [
@@ -104,7 +104,7 @@ def test_worked_example_values():
     np.testing.assert_allclose(out["fhat"][0, :, 0], g["fhat"], rtol=0)
 
 
-@pytest.mark.parametrize("prec", ["fp64", "fp32"])
+@pytest.mark.parametrize("prec", ["fp64", "fp32", "exact"])
 def test_host_buffers_match_device_buffers(prec):
     w = random_case(21, K=2, N=(3000, 211), L=(700, 700), R=19, n_lam=20, n_eps=2, M=2)
     a = run(w, P[prec])
@@ -210,3 +210,15 @@ def test_injected_allocation_failure_reports_enomem(monkeypatch):
     monkeypatch.delenv("KVDRO_TEST_FAIL_ALLOC")
     ctx = _loaded_ctx()
     kvdro.kvdro_destroy(ctx)
+
+
+def test_exact_mode_rejects_support_above_its_limit():
+    ctx = kvdro.kvdro_create(0)
+    try:
+        s = torch.tensor([1, 2, 3], dtype=torch.int32, device="cuda")
+        kvdro.kvdro_load_samples(ctx, 1, np.array([0, 3]), s, np.array([(1 << 22) + 1]))
+        ev = lambda p: kvdro.kvdro_eval_grid(ctx, p, 1, [3], 1, [1.0], 1, [0.0], 1, [2.0], [1.0])
+        assert _status(ev, kvdro.KVDRO_EXACT) == kvdro.KVDRO_EINVAL
+        ev(kvdro.KVDRO_FP64)  # the other modes accept it
+    finally:
+        kvdro.kvdro_destroy(ctx)
