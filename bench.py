@@ -48,6 +48,9 @@ TERMS_PER_CLK_PER_SM = LANE_OPS_PER_CLK_PER_SM / LANE_OPS_PER_TERM
 GRID_SOURCE = os.path.join(ROOT, "paper_2607_16892_gb300", "csrc", "grid.cu")
 PROFILE = os.path.join(ROOT, "profiles", "k_grid_f32_lognormal_k8_n1e5.md")
 LAUNCHES_PER_STEP = 6  # histogram, scan, expand, quantile gather, grid, argmin finalise
+# FP64 pipe bound of the native FP64 mode: per term one DFMA (2.0 per clk per SM) plus one DADD and
+# one max.f64 (1.7 per clk per SM each), measured on this GB300; nominal 1.25 TFLOP/s FP64.
+FP64_TERMS_PER_CLK_PER_SM = 1.0 / (1.0 / 2.0 + 2.0 / 1.7)
 
 
 def parse_args():
@@ -59,6 +62,9 @@ def parse_args():
     p.add_argument("--e2e-steps", type=int, default=30)
     p.add_argument("--cpu-seconds", type=float, default=10.0, help="target wall time of the CPU-baseline sample")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--drift-iterations", type=int, default=3)
+    p.add_argument("--suite", action="store_true",
+                   help="time every workload in each precision (one JSON line per case) instead of the contract line")
     return p.parse_args()
 
 
@@ -356,8 +362,59 @@ def run_reference(args):
     print(json.dumps(line), flush=True)
 
 
+def run_suite(args):
+    """Grid throughput on every workload and precision (device-resident samples, kernel time from
+    the library's CUDA events); plus a few iterations of the drifting-workload loop."""
+    import torch
+
+    from paper_2607_16892_gb300 import kvdro as kv
+    from paper_2607_16892_gb300.drift_loop import run as drift_run
+    from synth import WORKLOADS
+
+    dev = torch.device("cuda", 0)
+    props = torch.cuda.get_device_properties(dev)
+    peak32 = props.multi_processor_count * TERMS_PER_CLK_PER_SM * SM_MAX_MHZ_RECIPE * 1e6
+    peak64 = props.multi_processor_count * FP64_TERMS_PER_CLK_PER_SM * SM_MAX_MHZ_RECIPE * 1e6
+    names = {kv.KVDRO_FP32: "fp32", kv.KVDRO_FP64: "fp64", kv.KVDRO_EXACT: "exact"}
+    cases = [("lognormal_k3_n1e3", [kv.KVDRO_FP64, kv.KVDRO_EXACT, kv.KVDRO_FP32]),
+             ("lognormal_k8_n1e5", [kv.KVDRO_FP32, kv.KVDRO_EXACT, kv.KVDRO_FP64]),
+             ("heavytail_k16_n1e6", [kv.KVDRO_FP32, kv.KVDRO_EXACT]),
+             ("regimes_k8_n2e5", [kv.KVDRO_FP32, kv.KVDRO_EXACT])]
+    for name, precs in cases:
+        w = WORKLOADS[name]()
+        ctx = kv.kvdro_create(0)
+        d = torch.from_numpy(w.samples).to(dev)
+        M, E, K, R, NL = len(w.cp), len(w.eps), w.K, len(w.r), len(w.lam)
+        t0 = time.perf_counter()
+        kv.kvdro_load_samples(ctx, K, w.offsets, d, w.L, w.L_in)
+        load_ms = (time.perf_counter() - t0) * 1e3
+        for prec in precs:
+            r_idx = torch.empty((M, E, K), dtype=torch.int32, device=dev)
+            reps = 1 if (prec == kv.KVDRO_FP64 or w.terms() > 1e13) else 3
+            kv.kvdro_eval_grid(ctx, prec, R, w.r, NL, w.lam, E, w.eps, M, w.cp, w.cw, r_idx=r_idx)
+            ms = []
+            for _ in range(reps):
+                kv.kvdro_eval_grid(ctx, prec, R, w.r, NL, w.lam, E, w.eps, M, w.cp, w.cw, r_idx=r_idx)
+                ms.append(kv.kvdro_last_grid_ms(ctx))
+            grid_ms = float(np.median(ms))
+            rate = w.terms() / (grid_ms / 1e3)
+            peak = peak64 if prec == kv.KVDRO_FP64 else peak32
+            print(json.dumps({"suite": True, "workload": w.name, "precision": names[prec], "terms": w.terms(),
+                              "grid_ms": grid_ms, "terms_per_s": rate, "peak": peak, "frac": rate / peak,
+                              "load_sort_ms_wall": load_ms}), flush=True)
+        kv.kvdro_destroy(ctx)
+    recs = drift_run(iterations=args.drift_iterations, log=lambda *_: None)
+    for r in recs:
+        print(json.dumps({"suite": True, **{k: r[k] for k in ("workload", "iteration", "terms", "gpu_ms", "upload_ms",
+                                                                "sort_quantiles_ms", "eval_ms", "grid_kernel_ms",
+                                                                "terms_per_s")}}), flush=True)
+
+
 def main():
     args = parse_args()
+    if args.suite:
+        run_suite(args)
+        return
     if args.impl == "reference":
         run_reference(args)
     else:
