@@ -402,6 +402,20 @@ def run_suite(args):
             print(json.dumps({"suite": True, "workload": w.name, "precision": names[prec], "terms": w.terms(),
                               "grid_ms": grid_ms, "terms_per_s": rate, "peak": peak, "frac": rate / peak,
                               "load_sort_ms_wall": load_ms}), flush=True)
+        # not per term: the envelope mode (cells/s) and the exact dual over gamma ((m, e, k, r) cells/s)
+        for mode, label in ((kv.KVDRO_ENVELOPE, "envelope"), ("dual", "dual")):
+            r_idx = torch.empty((M, E, K), dtype=torch.int32, device=dev)
+            ms = []
+            for _ in range(3):
+                if mode == "dual":
+                    kv.kvdro_eval_dual(ctx, R, w.r, E, w.eps, M, w.cp, w.cw, r_idx=r_idx)
+                else:
+                    kv.kvdro_eval_grid(ctx, mode, R, w.r, NL, w.lam, E, w.eps, M, w.cp, w.cw, r_idx=r_idx)
+                ms.append(kv.kvdro_last_grid_ms(ctx))
+            grid_ms = float(np.median(ms[1:]))
+            cells = M * K * R * NL if mode != "dual" else M * E * K * R
+            print(json.dumps({"suite": True, "workload": w.name, "mode": label, "cells": cells, "grid_ms": grid_ms,
+                              "cells_per_s": cells / (grid_ms / 1e3)}), flush=True)
         kv.kvdro_destroy(ctx)
     recs = drift_run(iterations=args.drift_iterations, log=lambda *_: None)
     for r in recs:

@@ -56,9 +56,12 @@ typedef enum {
 typedef enum {
     KVDRO_FP32 = 0,      /* per-term arithmetic in FP32; sums folded into FP64 */
     KVDRO_FP64 = 1,      /* per-term arithmetic and sums in FP64 */
-    KVDRO_EXACT = 2      /* per-term FP32 decisions on exact integer thresholds, exact integer
+    KVDRO_EXACT = 2,     /* per-term FP32 decisions on exact integer thresholds, exact integer
                             counts and sample sums, combined once per cell in FP64; results
                             carry FP64 rounding only.  Needs every L_max <= 2^22. */
+    KVDRO_ENVELOPE = 3   /* not per term: each cell's sample sum from the sorted samples'
+                            cumulative counts and sums at its exact threshold, O(1) per cell,
+                            FP64 outputs with FP64 rounding only */
 } kvdro_precision;
 
 /* Create a context on CUDA device `device_ordinal`.  *out receives the handle (NULL on error). */
@@ -90,10 +93,10 @@ int kvdro_quantiles(kvdro_ctx* ctx, int32_t F, const double* fractiles, int32_t*
 
 /*
  * Evaluate the grid and reduce it.  Element type of S, cost and min_cost is float for
- * KVDRO_FP32 and double for KVDRO_FP64 and KVDRO_EXACT.
+ * KVDRO_FP32 and double for the other modes.
  *   R, r       host int32[R], 1 <= R <= 2^20; every r must satisfy L_in_k <= r <= L_in_k + L_k for
  *              every class (the reservation domain of Sec. 2.2).
- *   NL, lam    host double[NL], finite, >= 0; 1 <= NL <= 256 (FP32) or 128 (FP64, EXACT).
+ *   NL, lam    host double[NL], finite, >= 0; 1 <= NL <= 256 (FP32, ENVELOPE) or 128 (FP64, EXACT).
  *   E, eps     host double[E], finite, >= 0; 1 <= E <= 64.
  *   M, c_p,c_w host double[M] each, finite, >= 0; 1 <= M <= 65536.
  * Outputs (each may be NULL to skip it; host or device):
@@ -108,14 +111,34 @@ int kvdro_eval_grid(kvdro_ctx* ctx, int precision, int32_t R, const int32_t* r, 
                     int32_t E, const double* eps, int32_t M, const double* c_p, const double* c_w, void* S,
                     void* cost, int32_t* lam_idx, int32_t* r_idx, void* min_cost, double* fhat, void* stream);
 
+/*
+ * The exact worst-case expected cost, without restricting gamma to a grid: for every regime,
+ * radius, class and reservation, min over gamma >= 0 of gamma*eps + S(eta, gamma) (App. A,
+ * eq. app_kantorovich; the value of the epigraph LP of eq. app_lp, which equals the worst case
+ * over the Wasserstein ball by the strong duality of App. A Step 2).  The objective is convex
+ * and piecewise linear in gamma with its minimiser in [0, max(c_p, c_w)]; the library bisects on
+ * its right derivative (64 halvings) with every evaluation O(1) from the sorted samples'
+ * cumulative counts and sums, so results carry FP64 rounding only.
+ * Arguments as kvdro_eval_grid; outputs (each may be NULL; host or device):
+ *   cost       double [M][E][K][R]   the exact dual value
+ *   gamma      double [M][E][K][R]   a minimising gamma
+ *   r_idx      int32 [M][E][K]       lowest r index attaining the minimum (among costs equal to
+ *                                    2^-32 relative)
+ *   min_cost   double [M][E][K];  fhat  double [M][E][K]  as in kvdro_eval_grid
+ */
+int kvdro_eval_dual(kvdro_ctx* ctx, int32_t R, const int32_t* r, int32_t E, const double* eps, int32_t M,
+                    const double* c_p, const double* c_w, double* cost, double* gamma, int32_t* r_idx,
+                    double* min_cost, double* fhat, void* stream);
+
 /* Copy the sorted samples (class by class, ascending, int32[offsets[K]]) to `out` (host or device). */
 int kvdro_sorted_samples(const kvdro_ctx* ctx, int32_t* out, void* stream);
 
 /*
- * Device time, in milliseconds, of the grid-kernel launches of the last kvdro_eval_grid() call on
- * this context, measured with CUDA events recorded on that call's stream immediately before and
- * after them (the argmin finalisation and the output copies are outside).  Blocks until the
- * second event has completed.  KVDRO_ESTATE if no grid has been evaluated yet.
+ * Device time, in milliseconds, of the grid-kernel launches of the last kvdro_eval_grid() or
+ * kvdro_eval_dual() call on this context, measured with CUDA events recorded on that call's
+ * stream immediately before and after them (the argmin finalisation and the output copies are
+ * outside).  Blocks until the second event has completed.  KVDRO_ESTATE if nothing has been
+ * evaluated yet.
  */
 int kvdro_last_grid_ms(kvdro_ctx* ctx, float* ms);
 

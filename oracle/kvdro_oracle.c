@@ -255,3 +255,95 @@ int kvo_envelope_grid(const int64_t* C, const int64_t* Sx, int64_t stride, const
     free(th);
     return 0;
 }
+
+/* ---- the exact dual: min over gamma >= 0 of gamma eps + S(eta, gamma) --------------------------- */
+
+/* App. A eq. app_kantorovich without a grid.  g(gamma) is convex and piecewise linear (each sample's
+ * phi is a maximum of three lines in gamma: Q(eta,0) - gamma x, Q(eta,x), Q(eta,L) - gamma (L - x)),
+ * so its minimum over gamma >= 0 is at gamma = 0 or at a pairwise crossing of one sample's lines.
+ * Every candidate is evaluated with the envelope sum; the smallest value (first in candidate order on
+ * ties) is returned with its gamma.  `vals` holds the class's distinct sample values. */
+void kvo_exact_dual(const int64_t* C, const int64_t* Sx, int32_t L, int64_t N, const int32_t* vals, int64_t nvals,
+                    double eta, double eps, double cp, double cw, double* out_cost, double* out_gamma) {
+    const double q0 = kvo_Q(eta, 0.0, cp, cw), qL = kvo_Q(eta, (double)L, cp, cw);
+    double best = kvo_envelope_sum(C, Sx, L, eta, 0.0, cp, cw) / (double)N;  /* gamma = 0 */
+    double bg = 0.0;
+    for (int64_t i = 0; i < nvals; i++) {
+        const double x = (double)vals[i], qx = kvo_Q(eta, x, cp, cw);
+        double cand[3];
+        int nc = 0;
+        if (x > 0.0) cand[nc++] = (q0 - qx) / x;                       /* Q(0) - g x = Q(x)      */
+        if (x < (double)L) cand[nc++] = (qL - qx) / ((double)L - x);   /* Q(L) - g (L-x) = Q(x)  */
+        if (2.0 * x != (double)L) cand[nc++] = (q0 - qL) / (2.0 * x - (double)L); /* the two moved */
+        for (int c = 0; c < nc; c++) {
+            const double g = cand[c];
+            if (!(g > 0.0) || !isfinite(g)) continue;
+            const double v = g * eps + kvo_envelope_sum(C, Sx, L, eta, g, cp, cw) / (double)N;
+            if (v < best) { best = v; bg = g; }
+        }
+    }
+    *out_cost = best;
+    *out_gamma = bg;
+}
+
+typedef struct {
+    const int64_t* C;
+    const int64_t* Sx;
+    int64_t stride;
+    const int64_t* N;
+    const int32_t* L;
+    const int32_t* L_in;
+    const int32_t* vals;     /* distinct values, class k at vals_off[k] */
+    const int64_t* vals_off;
+    const int32_t* r;
+    const double* eps;
+    const double* cp;
+    const double* cw;
+    int32_t K, R, E;
+    double* cost;            /* [M][E][K][R] */
+    double* gamma;
+    int64_t begin, end;
+} dual_job;
+
+static void* dual_worker(void* arg) {
+    dual_job* j = (dual_job*)arg;
+    for (int64_t c = j->begin; c < j->end; c++) {
+        int64_t t = c;
+        const int ri = (int)(t % j->R); t /= j->R;
+        const int k = (int)(t % j->K); t /= j->K;
+        const int e = (int)(t % j->E);
+        const int m = (int)(t / j->E);
+        kvo_exact_dual(j->C + j->stride * k, j->Sx + j->stride * k, j->L[k], j->N[k], j->vals + j->vals_off[k],
+                       j->vals_off[k + 1] - j->vals_off[k], (double)j->r[ri] - (double)j->L_in[k], j->eps[e],
+                       j->cp[m], j->cw[m], &j->cost[c], &j->gamma[c]);
+    }
+    return NULL;
+}
+
+int kvo_exact_dual_grid(const int64_t* C, const int64_t* Sx, int64_t stride, const int64_t* N, const int32_t* L,
+                        const int32_t* L_in, const int32_t* vals, const int64_t* vals_off, const int32_t* r,
+                        const double* eps, const double* cp, const double* cw, int32_t M, int32_t E, int32_t K,
+                        int32_t R, double* cost, double* gamma, int nthreads) {
+    const int64_t ncells = (int64_t)M * E * K * R;
+    if (nthreads < 1) nthreads = 1;
+    if ((int64_t)nthreads > ncells) nthreads = ncells > 0 ? (int)ncells : 1;
+    dual_job* jobs = (dual_job*)malloc(sizeof(dual_job) * (size_t)nthreads);
+    pthread_t* th = (pthread_t*)malloc(sizeof(pthread_t) * (size_t)nthreads);
+    if (!jobs || !th) { free(jobs); free(th); return -2; }
+    int started = 0;
+    for (int t = 0; t < nthreads; t++) {
+        dual_job* j = &jobs[t];
+        j->C = C; j->Sx = Sx; j->stride = stride; j->N = N; j->L = L; j->L_in = L_in; j->vals = vals;
+        j->vals_off = vals_off; j->r = r; j->eps = eps; j->cp = cp; j->cw = cw; j->K = K; j->R = R; j->E = E;
+        j->cost = cost; j->gamma = gamma;
+        j->begin = ncells * t / nthreads;
+        j->end = ncells * (t + 1) / nthreads;
+        if (pthread_create(&th[t], NULL, dual_worker, j) != 0) break;
+        started++;
+    }
+    for (int t = 0; t < started; t++) pthread_join(th[t], NULL);
+    for (int t = started; t < nthreads; t++) dual_worker(&jobs[t]);
+    free(jobs);
+    free(th);
+    return 0;
+}

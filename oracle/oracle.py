@@ -68,6 +68,11 @@ def _load():
             lib.kvo_cumulative.argtypes = [P, i64, i32, P, P]
             lib.kvo_envelope_sum.restype = d
             lib.kvo_envelope_sum.argtypes = [P, P, i32, d, d, d, d]
+            lib.kvo_exact_dual.restype = None
+            lib.kvo_exact_dual.argtypes = [P, P, i32, i64, P, i64, d, d, d, d, P, P]
+            lib.kvo_exact_dual_grid.restype = ctypes.c_int
+            lib.kvo_exact_dual_grid.argtypes = [P, P, i64, P, P, P, P, P, P, P, P, P, i32, i32, i32, i32, P, P,
+                                                ctypes.c_int]
             lib.kvo_envelope_grid.restype = ctypes.c_int
             lib.kvo_envelope_grid.argtypes = [P, P, i64, P, P, P, P, P, P, P, i32, i32, i32, i32, P, ctypes.c_int]
             _lib = lib
@@ -170,6 +175,45 @@ def envelope_grid(w, threads: Optional[int] = None) -> np.ndarray:
     if rc != 0:
         raise RuntimeError("kvo_envelope_grid failed")
     return out
+
+
+def exact_dual_grid(w, threads: Optional[int] = None):
+    """cost[m, e, k, r] = min over gamma >= 0 of gamma eps_e + S(eta, gamma) (App. A,
+    eq. app_kantorovich without a grid) and a minimising gamma, by evaluating the convex
+    piecewise-linear objective at gamma = 0 and at every kink of every sample's supremum."""
+    a = _arrays(w)
+    K = w.K
+    stride = int(w.L.max()) + 1
+    C = np.zeros((K, stride), np.int64)
+    Sx = np.zeros((K, stride), np.int64)
+    vals, voff = [], [0]
+    for k in range(K):
+        c, s_ = cumulative(w, k)
+        C[k, :c.size] = c
+        Sx[k, :s_.size] = s_
+        u = np.unique(w.class_samples(k)).astype(np.int32)
+        vals.append(u)
+        voff.append(voff[-1] + u.size)
+    vals = np.ascontiguousarray(np.concatenate(vals), np.int32)
+    voff = np.ascontiguousarray(voff, np.int64)
+    N = np.ascontiguousarray(np.diff(w.offsets), np.int64)
+    eps = np.ascontiguousarray(w.eps, np.float64)
+    M, E, R = len(w.cp), len(w.eps), len(w.r)
+    cost = np.empty((M, E, K, R), np.float64)
+    gam = np.empty((M, E, K, R), np.float64)
+    rc = _load().kvo_exact_dual_grid(_p(C), _p(Sx), stride, _p(N), _p(a["L"]), _p(a["L_in"]), _p(vals), _p(voff),
+                                     _p(a["r"]), _p(eps), _p(a["cp"]), _p(a["cw"]), M, E, K, R, _p(cost), _p(gam),
+                                     int(threads or default_threads()))
+    if rc != 0:
+        raise RuntimeError("kvo_exact_dual_grid failed")
+    return cost, gam
+
+
+def solve_dual(w, threads: Optional[int] = None) -> Dict[str, np.ndarray]:
+    """The exact dual cost, a minimising gamma, the argmin over r, its minimum and Fhat(r*)."""
+    cost, gam = exact_dual_grid(w, threads)
+    r_idx, min_cost = argmin_r(cost)
+    return dict(cost=cost, gamma=gam, r_idx=r_idx, min_cost=min_cost, fhat=fhat_at(w, r_idx))
 
 
 # ---------------------------------------------------------------- epilogue

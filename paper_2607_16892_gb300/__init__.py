@@ -7,11 +7,13 @@ The computation lives in the CUDA library built from ``csrc/`` (C ABI in
 from . import kvdro  # noqa: F401
 from .kvdro import (  # noqa: F401
     KVDRO_FP32,
+    KVDRO_ENVELOPE,
     KVDRO_EXACT,
     KVDRO_FP64,
     KvdroError,
     kvdro_create,
     kvdro_destroy,
+    kvdro_eval_dual,
     kvdro_eval_grid,
     kvdro_last_error,
     kvdro_last_grid_ms,

@@ -17,7 +17,7 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 OUT_DIR = os.path.join(PKG, "_build")
 LIB = os.path.join(OUT_DIR, "libkvdro.so")
-SOURCES = ["api.cu", "sort.cu", "grid.cu", "noalloc.cu"]
+SOURCES = ["api.cu", "sort.cu", "grid.cu", "dual.cu", "noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -54,7 +54,7 @@ struct kvdro_ctx {
     std::vector<int64_t> off, pair_off, hist_off, N;
     std::vector<int32_t> L, Lin, hist_blocks, exp_blocks;
 
-    Buf sorted, pairs, hist, sumx, meta, errs, in_stage, grid_in, keys, cost64, out_stage, ranks;
+    Buf sorted, pairs, hist, csum, sumx, meta, errs, in_stage, grid_in, keys, cost64, out_stage, ranks;
     void* pin = nullptr;  // pinned host staging
     size_t pin_bytes = 0;
     cudaEvent_t pin_free = nullptr;  // completes when the last copy out of `pin` is done
@@ -208,7 +208,8 @@ int kvdro_create(kvdro_ctx** out, int device_ordinal) {
     DeviceGuard g(device_ordinal);
     if (!g.ok || kvdro::grid_prepare(Prec::F32) != cudaSuccess || kvdro::grid_prepare(Prec::F64) != cudaSuccess ||
         cudaEventCreateWithFlags(&ctx->pin_free, cudaEventDisableTiming) != cudaSuccess ||
-        kvdro::grid_prepare(Prec::EXACT) != cudaSuccess || cudaEventCreate(&ctx->grid_t0) != cudaSuccess ||
+        kvdro::grid_prepare(Prec::EXACT) != cudaSuccess || kvdro::grid_prepare(Prec::ENVELOPE) != cudaSuccess ||
+        cudaEventCreate(&ctx->grid_t0) != cudaSuccess ||
         cudaEventCreate(&ctx->grid_t1) != cudaSuccess) {
         cudaGetLastError();
         delete ctx;
@@ -223,7 +224,7 @@ int kvdro_destroy(kvdro_ctx* ctx) {
     DeviceGuard g(ctx->device);
     if (ctx->last_stream) cudaStreamSynchronize(ctx->last_stream);
     cudaDeviceSynchronize();
-    for (Buf* b : {&ctx->sorted, &ctx->pairs, &ctx->hist, &ctx->sumx, &ctx->meta, &ctx->errs, &ctx->in_stage,
+    for (Buf* b : {&ctx->sorted, &ctx->pairs, &ctx->hist, &ctx->csum, &ctx->sumx, &ctx->meta, &ctx->errs, &ctx->in_stage,
                    &ctx->grid_in, &ctx->keys, &ctx->cost64, &ctx->out_stage, &ctx->ranks})
         release(*b);
     if (ctx->pin) cudaFreeHost(ctx->pin);
@@ -290,6 +291,7 @@ int kvdro_load_samples(kvdro_ctx* ctx, int32_t K, const int64_t* offsets, const 
     if ((rc = ensure(ctx, ctx->sorted, (size_t)ctx->total * 4))) return rc;
     if ((rc = ensure(ctx, ctx->pairs, (size_t)ctx->pair_total * 8))) return rc;
     if ((rc = ensure(ctx, ctx->hist, (size_t)ctx->hist_total * 4))) return rc;
+    if ((rc = ensure(ctx, ctx->csum, (size_t)ctx->hist_total * 8))) return rc;
     if ((rc = ensure(ctx, ctx->sumx, (size_t)K * 8))) return rc;
     if ((rc = ensure(ctx, ctx->errs, 2 * sizeof(int32_t)))) return rc;
     const size_t meta_bytes = (size_t)(K + 1) * 8 * 3 + (size_t)K * 8 + (size_t)K * 4 * 2 + (size_t)(K + 1) * 4 * 2 + 64;
@@ -337,6 +339,7 @@ int kvdro_load_samples(kvdro_ctx* ctx, int32_t K, const int64_t* offsets, const 
     a.hist_blocks = ctx->d_hist_blocks;
     a.exp_blocks = ctx->d_exp_blocks;
     a.hist = static_cast<int32_t*>(ctx->hist.p);
+    a.csum = static_cast<int64_t*>(ctx->csum.p);
     a.sumx = static_cast<int64_t*>(ctx->sumx.p);
     a.sorted = static_cast<int32_t*>(ctx->sorted.p);
     a.pairs = static_cast<float2*>(ctx->pairs.p);
@@ -407,10 +410,12 @@ int kvdro_eval_grid(kvdro_ctx* ctx, int precision, int32_t R, const int32_t* r, 
     if (!ctx) return KVDRO_EINVAL;
     ctx->err.clear();
     if (!ctx->loaded) return fail(ctx, KVDRO_ESTATE, "no samples loaded");
-    if (precision != KVDRO_FP32 && precision != KVDRO_FP64 && precision != KVDRO_EXACT)
-        return fail(ctx, KVDRO_EINVAL, "precision must be KVDRO_FP32, KVDRO_FP64 or KVDRO_EXACT");
-    const Prec P = precision == KVDRO_FP32 ? Prec::F32 : precision == KVDRO_FP64 ? Prec::F64 : Prec::EXACT;
-    const int32_t maxNL = P == Prec::F32 ? kMaxNLf32 : kMaxNLf64;
+    if (precision != KVDRO_FP32 && precision != KVDRO_FP64 && precision != KVDRO_EXACT && precision != KVDRO_ENVELOPE)
+        return fail(ctx, KVDRO_EINVAL, "precision must be KVDRO_FP32, KVDRO_FP64, KVDRO_EXACT or KVDRO_ENVELOPE");
+    const Prec P = precision == KVDRO_FP32 ? Prec::F32
+                 : precision == KVDRO_FP64 ? Prec::F64
+                 : precision == KVDRO_EXACT ? Prec::EXACT : Prec::ENVELOPE;
+    const int32_t maxNL = (P == Prec::F32 || P == Prec::ENVELOPE) ? kMaxNLf32 : kMaxNLf64;
     if (P == Prec::EXACT)
         for (int32_t k = 0; k < ctx->K; k++)
             if (ctx->L[k] > kvdro::kExactMaxL)
@@ -507,6 +512,7 @@ int kvdro_eval_grid(kvdro_ctx* ctx, int precision, int32_t R, const int32_t* r, 
     a.L = ctx->d_L;
     a.L_in = ctx->d_Lin;
     a.cdf = static_cast<const int32_t*>(ctx->hist.p);
+    a.csum = static_cast<const int64_t*>(ctx->csum.p);
     a.hist_off = ctx->d_hist_off;
     a.r = d_r;
     a.lam = d_lam;
@@ -558,6 +564,136 @@ int kvdro_eval_grid(kvdro_ctx* ctx, int precision, int32_t R, const int32_t* r, 
                 KV_CUDA(cudaMemcpyAsync(x.user, x.dev, x.bytes, cudaMemcpyDeviceToHost, s), "copying results");
         KV_CUDA(cudaStreamSynchronize(s), "copying results");
         return check_kernel_errors(ctx, s);
+    }
+    return KVDRO_OK;
+}
+
+int kvdro_eval_dual(kvdro_ctx* ctx, int32_t R, const int32_t* r, int32_t E, const double* eps, int32_t M,
+                    const double* c_p, const double* c_w, double* cost, double* gamma, int32_t* r_idx,
+                    double* min_cost, double* fhat, void* stream) {
+    if (!ctx) return KVDRO_EINVAL;
+    ctx->err.clear();
+    if (!ctx->loaded) return fail(ctx, KVDRO_ESTATE, "no samples loaded");
+    if (R < 1 || R > kMaxR) return fail(ctx, KVDRO_EINVAL, "R = %d outside [1, 2^20]", R);
+    if (E < 1 || E > kMaxE) return fail(ctx, KVDRO_EINVAL, "E = %d outside [1, %d]", E, kMaxE);
+    if (M < 1 || M > kMaxM) return fail(ctx, KVDRO_EINVAL, "M = %d outside [1, %d]", M, kMaxM);
+    if (!r || !eps || !c_p || !c_w) return fail(ctx, KVDRO_EINVAL, "r, eps, c_p and c_w are required");
+    if (!finite_nonneg(eps, E)) return fail(ctx, KVDRO_EINVAL, "eps must be finite and >= 0");
+    if (!finite_nonneg(c_p, M) || !finite_nonneg(c_w, M)) return fail(ctx, KVDRO_EINVAL, "costs must be finite and >= 0");
+    for (int32_t i = 0; i < R; i++)
+        for (int32_t k = 0; k < ctx->K; k++)
+            if ((int64_t)r[i] < ctx->Lin[k] || (int64_t)r[i] > (int64_t)ctx->Lin[k] + ctx->L[k])
+                return fail(ctx, KVDRO_EINVAL, "r[%d] = %d outside [L_in, L_in + L_max] of class %d", i, r[i], k);
+    const int64_t cells = (int64_t)M * E * ctx->K * R;
+    const int64_t rows = (int64_t)M * E * ctx->K;
+    if (cells > 0x7fffffffLL * 256LL) return fail(ctx, KVDRO_EINVAL, "grid too large");
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    DeviceGuard g(ctx->device);
+    if (!g.ok) return fail(ctx, KVDRO_ECUDA, "cannot select device %d", ctx->device);
+    ctx->last_stream = s;
+
+    const size_t gbytes = align_up((size_t)R * 4, 8) + 8 * ((size_t)E + 2 * (size_t)M);
+    int rc;
+    if ((rc = ensure(ctx, ctx->grid_in, gbytes))) return rc;
+    void* hp;
+    if ((rc = pinned(ctx, gbytes, &hp))) return rc;
+    char* h = static_cast<char*>(hp);
+    char* d = static_cast<char*>(ctx->grid_in.p);
+    size_t o = 0;
+    auto put = [&](const void* src, size_t bytes) {
+        std::memcpy(h + o, src, bytes);
+        void* dv = d + o;
+        o = align_up(o + bytes, 8);
+        return dv;
+    };
+    const int32_t* d_r = static_cast<const int32_t*>(put(r, (size_t)R * 4));
+    const double* d_eps = static_cast<const double*>(put(eps, (size_t)E * 8));
+    const double* d_cp = static_cast<const double*>(put(c_p, (size_t)M * 8));
+    const double* d_cw = static_cast<const double*>(put(c_w, (size_t)M * 8));
+    KV_CUDA(cudaMemcpyAsync(ctx->grid_in.p, hp, o, cudaMemcpyHostToDevice, s), "uploading the grid");
+    KV_CUDA(cudaEventRecord(ctx->pin_free, s), "recording staging event");
+
+    struct Out {
+        void* user;
+        size_t bytes;
+        bool host;
+        void* dev;
+    };
+    Out outs[5] = {{cost, (size_t)cells * 8, false, nullptr},
+                   {gamma, (size_t)cells * 8, false, nullptr},
+                   {r_idx, (size_t)rows * 4, false, nullptr},
+                   {min_cost, (size_t)rows * 8, false, nullptr},
+                   {fhat, (size_t)rows * 8, false, nullptr}};
+    size_t stage_bytes = 0;
+    for (Out& x : outs) {
+        if (!x.user) continue;
+        x.host = !is_device_ptr(x.user);
+        if (x.host) stage_bytes += align_up(x.bytes, 256);
+        else x.dev = x.user;
+    }
+    if (stage_bytes) {
+        if ((rc = ensure(ctx, ctx->out_stage, stage_bytes))) return rc;
+        size_t so = 0;
+        for (Out& x : outs)
+            if (x.user && x.host) {
+                x.dev = static_cast<char*>(ctx->out_stage.p) + so;
+                so += align_up(x.bytes, 256);
+            }
+    }
+    void* cost_dev = outs[0].dev;
+    if (!cost_dev) {
+        if ((rc = ensure(ctx, ctx->cost64, (size_t)cells * 8))) return rc;
+        cost_dev = ctx->cost64.p;
+    }
+    if ((rc = ensure(ctx, ctx->keys, (size_t)rows * 8))) return rc;
+    KV_CUDA(cudaMemsetAsync(ctx->keys.p, 0xFF, (size_t)rows * 8, s), "clearing argmin keys");
+
+    kvdro::DualArgs a;
+    a.cdf = static_cast<const int32_t*>(ctx->hist.p);
+    a.csum = static_cast<const int64_t*>(ctx->csum.p);
+    a.hist_off = ctx->d_hist_off;
+    a.N = ctx->d_N;
+    a.sumx = static_cast<const int64_t*>(ctx->sumx.p);
+    a.L = ctx->d_L;
+    a.L_in = ctx->d_Lin;
+    a.r = d_r;
+    a.eps = d_eps;
+    a.cp = d_cp;
+    a.cw = d_cw;
+    a.K = ctx->K;
+    a.R = R;
+    a.E = E;
+    a.M = M;
+    a.cost = static_cast<double*>(cost_dev);
+    a.gamma = static_cast<double*>(outs[1].dev);
+    a.keys = static_cast<unsigned long long*>(ctx->keys.p);
+    ctx->grid_timed = false;
+    KV_CUDA(cudaEventRecord(ctx->grid_t0, s), "recording dual start");
+    KV_CUDA(kvdro::launch_dual(a, s), "dual kernel");
+    KV_CUDA(cudaEventRecord(ctx->grid_t1, s), "recording dual end");
+    ctx->grid_timed = true;
+
+    kvdro::FinalizeArgs fa;
+    fa.keys = a.keys;
+    fa.cost = cost_dev;
+    fa.r = d_r;
+    fa.L_in = ctx->d_Lin;
+    fa.N = ctx->d_N;
+    fa.cdf = a.cdf;
+    fa.hist_off = ctx->d_hist_off;
+    fa.K = ctx->K;
+    fa.R = R;
+    fa.E = E;
+    fa.M = M;
+    fa.r_idx = static_cast<int32_t*>(outs[2].dev);
+    fa.min_cost = outs[3].dev;
+    fa.fhat = static_cast<double*>(outs[4].dev);
+    if (fa.r_idx || fa.min_cost || fa.fhat) KV_CUDA(kvdro::launch_finalize(Prec::F64, fa, s), "finalize kernel");
+    if (stage_bytes) {
+        for (Out& x : outs)
+            if (x.user && x.host)
+                KV_CUDA(cudaMemcpyAsync(x.user, x.dev, x.bytes, cudaMemcpyDeviceToHost, s), "copying results");
+        KV_CUDA(cudaStreamSynchronize(s), "copying results");
     }
     return KVDRO_OK;
 }

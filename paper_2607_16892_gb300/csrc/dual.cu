@@ -1,0 +1,117 @@
+// The exact dual value of App. A (eq. app_kantorovich, gamma >= 0 not restricted to a grid):
+//   cost(eta, eps) = min_{gamma >= 0} g(gamma),  g(gamma) = gamma eps + S(eta, gamma).
+// g is convex and piecewise linear in gamma (each sample's supremum is a maximum of lines in
+// gamma).  For gamma >= max(c_p, c_w) moving mass never pays and S is the empirical cost, so g
+// rises with slope eps and the minimiser lies in [0, max(c_p, c_w)].  One thread per
+// (regime, radius, class, reservation) bisects on the sign of the right derivative; every
+// evaluation of S and of its derivative is O(1) from the class's cumulative counts and sums:
+// with mu = min(gamma, c_p), nu = min(gamma, c_w), kappa = mu + nu and
+// d = (c_p - mu) L - (c_p + c_w) eta, the samples with a positive excess kappa x + d are x >= t
+// for an integer threshold t, and
+//   N S = N c_w eta - nu sum(x) + kappa sum_{x >= t} x + d #{x >= t}.
+#include <float.h>
+#include <math.h>
+
+#include "kvdro_internal.cuh"
+
+namespace kvdro {
+namespace {
+
+constexpr int kDualThreads = 256;
+constexpr int kBisections = 64;
+
+struct ClassView {
+    const int32_t* C;   // cumulative counts, L + 1 entries
+    const int64_t* CS;  // cumulative sums
+    int64_t N;
+    int64_t sumx;
+    int32_t L;
+};
+
+// count and sum of the samples with x >= t (t clamped to [0, L + 1])
+__device__ __forceinline__ void tail(const ClassView& c, int64_t t, int64_t& cnt, int64_t& sum) {
+    const int64_t below_n = t >= 1 ? (int64_t)c.C[t - 1] : 0;
+    const int64_t below_s = t >= 1 ? c.CS[t - 1] : 0;
+    cnt = c.N - below_n;
+    sum = c.sumx - below_s;
+}
+
+__device__ __forceinline__ int64_t threshold(double kap, double d, int32_t L) {
+    if (kap > 0.0) {
+        const double xs = floor(-d / kap) + 1.0;
+        return xs <= 0.0 ? 0 : (xs >= (double)L + 1.0 ? (int64_t)L + 1 : (int64_t)xs);
+    }
+    return d > 0.0 ? 0 : (int64_t)L + 1;
+}
+
+// g(gamma) and its right derivative.
+__device__ __forceinline__ void g_and_slope(const ClassView& c, double eta, double cp, double cw, double eps, double gam,
+                                            double& g, double& slope) {
+    const double mu = fmin(gam, cp), nu = fmin(gam, cw), kap = mu + nu;
+    const double dmu = gam < cp ? 1.0 : 0.0, dnu = gam < cw ? 1.0 : 0.0;
+    const double L = (double)c.L, N = (double)c.N;
+    const double d = (cp - mu) * L - (cp + cw) * eta;
+    int64_t cnt, sum;
+    tail(c, threshold(kap, d, c.L), cnt, sum);
+    const double tot = N * cw * eta - nu * (double)c.sumx + kap * (double)sum + d * (double)cnt;
+    g = gam * eps + tot / N;
+    // right derivative: the active set just above gamma is the one at gamma up to samples whose
+    // excess is exactly zero, which change the value by nothing and the slope only at a kink
+    slope = eps + (-dnu * (double)c.sumx + (dmu + dnu) * (double)sum - dmu * L * (double)cnt) / N;
+}
+
+__global__ void __launch_bounds__(kDualThreads) k_dual(const DualArgs a) {
+    const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    const int64_t total = (int64_t)a.M * a.E * a.K * a.R;
+    if (i >= total) return;
+    int64_t t = i;
+    const int ri = (int)(t % a.R);
+    t /= a.R;
+    const int k = (int)(t % a.K);
+    t /= a.K;
+    const int e = (int)(t % a.E);
+    const int m = (int)(t / a.E);
+    ClassView c;
+    c.C = a.cdf + a.hist_off[k];
+    c.CS = a.csum + a.hist_off[k];
+    c.N = a.N[k];
+    c.sumx = a.sumx[k];
+    c.L = a.L[k];
+    const double cp = a.cp[m], cw = a.cw[m], eps = a.eps[e];
+    const double eta = (double)a.r[ri] - (double)a.L_in[k];
+    double lo = 0.0, hi = fmax(cp, cw), g_lo, s_lo, g_hi, s_hi;
+    g_and_slope(c, eta, cp, cw, eps, lo, g_lo, s_lo);
+    double best_g = g_lo, best_gam = lo;
+    if (s_lo < 0.0 && hi > 0.0) {
+        g_and_slope(c, eta, cp, cw, eps, hi, g_hi, s_hi);
+        for (int it = 0; it < kBisections; it++) {
+            const double mid = 0.5 * (lo + hi);
+            if (!(mid > lo && mid < hi)) break;
+            double gm, sm;
+            g_and_slope(c, eta, cp, cw, eps, mid, gm, sm);
+            if (sm >= 0.0) { hi = mid; g_hi = gm; }
+            else { lo = mid; g_lo = gm; }
+        }
+        // g is linear between kinks: the better end of the final bracket is the minimum
+        if (g_hi < g_lo) { best_g = g_hi; best_gam = hi; }
+        else { best_g = g_lo; best_gam = lo; }
+    }
+    const size_t row = ((size_t)m * a.E + e) * a.K + k;
+    if (a.cost) a.cost[row * a.R + ri] = best_g;
+    if (a.gamma) a.gamma[row * a.R + ri] = best_gam;
+    const unsigned long long key =
+        ((unsigned long long)__double_as_longlong(best_g > 0.0 ? best_g : 0.0) & ~0xFFFFFull) | (unsigned long long)ri;
+    atomicMin(a.keys + row, key);
+}
+
+}  // namespace
+
+cudaError_t launch_dual(const DualArgs& a, cudaStream_t s) {
+    const int64_t total = (int64_t)a.M * a.E * a.K * a.R;
+    const int64_t blocks = (total + kDualThreads - 1) / kDualThreads;
+    if (blocks <= 0 || blocks > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
+    k_dual<<<(unsigned)blocks, kDualThreads, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
+}  // namespace kvdro

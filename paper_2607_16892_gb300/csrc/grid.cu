@@ -199,6 +199,48 @@ __host__ __device__ inline SmemLayout smem_layout(int RG, int TR, int NLpad, int
     return L;
 }
 
+// Epilogue of one CTA: for each of its (r, eps) pairs, the minimum over lam of lam * eps + S
+// (lowest index on ties), the cost and lam index outputs, and the argmin over r through a 64-bit
+// atomicMin key (FP32: cost bits and r index; otherwise the cost's double bits truncated to 44
+// bits, order-preserving for non-negative values, with the r index in the low 20 bits).
+template <bool F32OUT>
+__device__ __forceinline__ void cta_epilogue(const GridArgs& a, const double* s_S, const double* s_lam,
+                                             const double* s_eps, int stride, int rl_count, int r_cta0, int m, int k) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
+    for (int p = warp; p < rl_count * a.E; p += nwarps) {
+        const int rl = p / a.E, e = p % a.E;
+        const int ri = r_cta0 + rl;
+        if (ri >= a.R) continue;
+        double best = DBL_MAX;
+        int bj = 0x7fffffff;
+        for (int j = lane; j < a.NL; j += 32) {
+            const double v = __dadd_rn(__dmul_rn(s_lam[j], s_eps[e]), s_S[rl * stride + j]);
+            if (v < best) { best = v; bj = j; }
+        }
+#pragma unroll
+        for (int o = 16; o; o >>= 1) {
+            const double ov = __shfl_xor_sync(0xffffffffu, best, o);
+            const int oj = __shfl_xor_sync(0xffffffffu, bj, o);
+            if (ov < best || (ov == best && oj < bj)) { best = ov; bj = oj; }
+        }
+        if (lane == 0) {
+            const size_t row = ((size_t)m * a.E + e) * a.K + k;
+            const size_t o = row * a.R + ri;
+            u64 key;
+            if constexpr (F32OUT) {
+                const float cf = (float)best;
+                if (a.cost_out) static_cast<float*>(a.cost_out)[o] = cf;
+                key = ((u64)__float_as_uint(cf > 0.f ? cf : 0.f) << 32) | (u64)(uint32_t)ri;
+            } else {
+                static_cast<double*>(a.cost_out)[o] = best;
+                key = ((u64)__double_as_longlong(best > 0.0 ? best : 0.0) & ~0xFFFFFull) | (u64)ri;
+            }
+            if (a.lam_idx_out) a.lam_idx_out[o] = bj;
+            atomicMin(a.keys + row, key);
+        }
+    }
+}
+
 // ---------------------------------------------------------------- the grid kernel
 
 template <class C>
@@ -521,42 +563,59 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
     }
     __syncthreads();
 
-    // Epilogue: for each (r, eps) of the CTA, the minimum over lam (lowest index on ties), the
-    // cost and lam index outputs, and the argmin over r through a 64-bit atomicMin key.
-    const int rl_count = a.RG * TR;
-    for (int p = warp; p < rl_count * a.E; p += nwarps) {
-        const int rl = p / a.E, e = p % a.E;
+    cta_epilogue<P == Prec::F32>(a, s_S, s_lam, s_eps, NLpad, a.RG * TR, r_cta0, m, k);
+}
+
+// The same cells in O(1) each from the class's cumulative counts C[v] = #{x <= v} and sums
+// CS[v] = sum_{x <= v} x: the samples with kappa x + d > 0 are exactly x >= t for the integer
+// threshold t, so sum_n max(kappa x_n + d, 0) = kappa (sum - CS[t-1]) + d (N - C[t-1]).
+constexpr int kEnvR = 8;          // r values per CTA
+constexpr int kEnvThreads = 256;
+
+__global__ void __launch_bounds__(kEnvThreads) k_envelope(const GridArgs a) {
+    extern __shared__ __align__(16) double esm[];
+    double* s_lam = esm;
+    double* s_eps = s_lam + a.NL;
+    double* s_S = s_eps + a.E;
+    int b = blockIdx.x;
+    const int rb = b % a.r_blocks;
+    b /= a.r_blocks;
+    const int k = b % a.K;
+    const int m = a.m0 + b / a.K;
+    const int r_cta0 = rb * kEnvR;
+    for (int i = threadIdx.x; i < a.NL; i += blockDim.x) s_lam[i] = a.lam[i];
+    for (int i = threadIdx.x; i < a.E; i += blockDim.x) s_eps[i] = a.eps[i];
+    __syncthreads();
+    const double cp = a.cp[m], cw = a.cw[m];
+    const int32_t Lk = a.L[k];
+    const int64_t Nk = a.N[k];
+    const double N = (double)Nk, sumx = (double)a.sumx[k];
+    const int32_t* C = a.cdf + a.hist_off[k];
+    const int64_t* CS = a.csum + a.hist_off[k];
+    for (int cell = threadIdx.x; cell < kEnvR * a.NL; cell += blockDim.x) {
+        const int rl = cell / a.NL, j = cell % a.NL;
         const int ri = r_cta0 + rl;
         if (ri >= a.R) continue;
-        double best = DBL_MAX;
-        int bj = 0x7fffffff;
-        for (int j = lane; j < a.NL; j += 32) {
-            const double v = __dadd_rn(__dmul_rn(s_lam[j], s_eps[e]), s_S[rl * NLpad + j]);
-            if (v < best) { best = v; bj = j; }
+        const double eta = (double)a.r[ri] - (double)a.L_in[k];
+        const double lam = s_lam[j];
+        const double mu = fmin(lam, cp), nu = fmin(lam, cw), kap = mu + nu;
+        const double d = (cp - mu) * (double)Lk - (cp + cw) * eta;
+        int64_t t;  // first active sample value, clamped to [0, L + 1]
+        if (kap > 0.0) {
+            const double xs = floor(-d / kap) + 1.0;
+            t = xs <= 0.0 ? 0 : (xs >= (double)Lk + 1.0 ? (int64_t)Lk + 1 : (int64_t)xs);
+        } else {
+            t = d > 0.0 ? 0 : (int64_t)Lk + 1;
         }
-#pragma unroll
-        for (int o = 16; o; o >>= 1) {
-            const double ov = __shfl_xor_sync(0xffffffffu, best, o);
-            const int oj = __shfl_xor_sync(0xffffffffu, bj, o);
-            if (ov < best || (ov == best && oj < bj)) { best = ov; bj = oj; }
-        }
-        if (lane == 0) {
-            const size_t row = ((size_t)m * a.E + e) * a.K + k;
-            const size_t o = row * a.R + ri;
-            u64 key;
-            if constexpr (P == Prec::F32) {
-                const float cf = (float)best;
-                if (a.cost_out) static_cast<float*>(a.cost_out)[o] = cf;
-                key = ((u64)__float_as_uint(cf > 0.f ? cf : 0.f) << 32) | (u64)(uint32_t)ri;
-            } else {
-                static_cast<double*>(a.cost_out)[o] = best;
-                // order-preserving for non-negative doubles; keeps 32 mantissa bits, index in the low 20
-                key = ((u64)__double_as_longlong(best > 0.0 ? best : 0.0) & ~0xFFFFFull) | (u64)ri;
-            }
-            if (a.lam_idx_out) a.lam_idx_out[o] = bj;
-            atomicMin(a.keys + row, key);
-        }
+        const int64_t below_n = t >= 1 ? (int64_t)C[t - 1] : 0;
+        const int64_t below_s = t >= 1 ? CS[t - 1] : 0;
+        const double tot = N * cw * eta - nu * sumx + kap * (double)(a.sumx[k] - below_s) + d * (double)(Nk - below_n);
+        const double S = tot / N;
+        s_S[rl * a.NL + j] = S;
+        if (a.S_out) static_cast<double*>(a.S_out)[(((size_t)m * a.K + k) * a.R + ri) * a.NL + j] = S;
     }
+    __syncthreads();
+    cta_epilogue<false>(a, s_S, s_lam, s_eps, a.NL, kEnvR, r_cta0, m, k);
 }
 
 template <Prec P>
@@ -598,6 +657,16 @@ GridShape shape_for(int variant, int32_t R, int32_t NL, int32_t E) {
 }
 
 GridShape grid_shape(Prec p, int32_t R, int32_t NL, int32_t E) {
+    if (p == Prec::ENVELOPE) {
+        GridShape sh;
+        sh.variant = 4;
+        sh.LT = 1;
+        sh.RG = 1;
+        sh.threads = kEnvThreads;
+        sh.r_blocks = (R + kEnvR - 1) / kEnvR;
+        sh.smem = 8 * ((size_t)NL + E + (size_t)kEnvR * NL);
+        return sh;
+    }
     if (p == Prec::F64) return shape_for<CfgF64>(2, R, NL, E);
     if (p == Prec::EXACT) return shape_for<CfgExact>(3, R, NL, E);
     if (NL <= kWarpsTarget * CfgF32::TL) return shape_for<CfgF32>(0, R, NL, E);
@@ -609,6 +678,9 @@ cudaError_t grid_prepare(Prec p) {
     const int mx = (int)(smem_layout(16, 2, 256, 64).total + 4096);
     if (p == Prec::F64) return cudaFuncSetAttribute(k_grid<CfgF64>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
     if (p == Prec::EXACT) return cudaFuncSetAttribute(k_grid<CfgExact>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
+    if (p == Prec::ENVELOPE)
+        return cudaFuncSetAttribute(k_envelope, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    (int)(8 * (256 + 64 + (size_t)kEnvR * 256)));
     cudaError_t e = cudaFuncSetAttribute(k_grid<CfgF32>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
     if (e != cudaSuccess) return e;
     return cudaFuncSetAttribute(k_grid<CfgF32Wide>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
@@ -620,7 +692,8 @@ cudaError_t launch_grid(Prec p, const GridShape& sh, GridArgs a, cudaStream_t s)
     a.r_blocks = sh.r_blocks;
     const int64_t nblocks = (int64_t)a.m_count * a.K * a.r_blocks;
     if (nblocks <= 0 || nblocks > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
-    if (p == Prec::F64) k_grid<CfgF64><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
+    if (p == Prec::ENVELOPE) k_envelope<<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
+    else if (p == Prec::F64) k_grid<CfgF64><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
     else if (p == Prec::EXACT) k_grid<CfgExact><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
     else if (sh.variant == 0) k_grid<CfgF32><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
     else k_grid<CfgF32Wide><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);

@@ -24,6 +24,7 @@ struct SortArgs {
     const int32_t* hist_blocks; // [K+1] prefix of histogram blocks per class
     const int32_t* exp_blocks;  // [K+1] prefix of expand blocks per class
     int32_t* hist;              // [hist_off[K]] counts, then cumulative counts (in place)
+    int64_t* csum;              // [hist_off[K]] cumulative sums sum_{x <= v} x, or nullptr to skip
     int64_t* sumx;              // [K] sum of samples per class
     int32_t* sorted;            // [offsets[K]]
     float2* pairs;              // [pair_off[K]]
@@ -40,7 +41,8 @@ cudaError_t launch_gather_quantiles(const int32_t* sorted, const int64_t* offset
 
 // F32: per-term FP32 excess sums folded into FP64.  F64: per-term FP64.  EXACT: per-term FP32
 // threshold decisions with exact integer count and sample-sum accumulation, combined in FP64.
-enum class Prec { F32 = 0, F64 = 1, EXACT = 2 };
+// ENVELOPE: the same sums in O(1) per cell from cumulative counts and sums (not per term).
+enum class Prec { F32 = 0, F64 = 1, EXACT = 2, ENVELOPE = 3 };
 constexpr int32_t kExactMaxL = 1 << 22;  // EXACT needs 2 * L < 2^23 per fold of two samples
 
 struct GridArgs {
@@ -51,6 +53,7 @@ struct GridArgs {
     const int32_t* L;           // [K]
     const int32_t* L_in;        // [K]
     const int32_t* cdf;         // cumulative counts, class k at hist_off[k]
+    const int64_t* csum;        // cumulative sample sums, same layout (envelope mode)
     const int64_t* hist_off;    // [K+1]
     const int32_t* r;           // [R]
     const double* lam;          // [NL]
@@ -98,5 +101,25 @@ cudaError_t grid_prepare(Prec p);             // per-device attribute setup of e
 // Launches over regimes [a.m0, a.m0 + a.m_count); fills a.LT, a.RG, a.r_blocks from `sh`.
 cudaError_t launch_grid(Prec p, const GridShape& sh, GridArgs a, cudaStream_t s);
 cudaError_t launch_finalize(Prec p, const FinalizeArgs& a, cudaStream_t s);
+
+// dual.cu: exact minimisation over gamma >= 0 per (regime, radius, class, reservation)
+struct DualArgs {
+    const int32_t* cdf;         // cumulative counts, class k at hist_off[k]
+    const int64_t* csum;        // cumulative sums, same layout
+    const int64_t* hist_off;    // [K+1]
+    const int64_t* N;           // [K]
+    const int64_t* sumx;        // [K]
+    const int32_t* L;           // [K]
+    const int32_t* L_in;        // [K]
+    const int32_t* r;           // [R]
+    const double* eps;          // [E]
+    const double* cp;           // [M]
+    const double* cw;           // [M]
+    int32_t K, R, E, M;
+    double* cost;               // [M][E][K][R] (needed for min_cost)
+    double* gamma;              // optional [M][E][K][R]
+    unsigned long long* keys;   // [M][E][K], initialised to all ones
+};
+cudaError_t launch_dual(const DualArgs& a, cudaStream_t s);
 
 }  // namespace kvdro

@@ -234,6 +234,7 @@ extern "C" int kvdro_eval_grid_noalloc(int32_t K, const int64_t* offsets, const 
     sa.hist_blocks = mt.hist_blocks;
     sa.exp_blocks = mt.exp_blocks;
     sa.hist = reinterpret_cast<int32_t*>(S + o_hist);
+    sa.csum = nullptr;  // cumulative sums are not needed here
     sa.sumx = reinterpret_cast<int64_t*>(S + o_sumx);
     sa.sorted = reinterpret_cast<int32_t*>(S + o_sorted);
     sa.pairs = reinterpret_cast<float2*>(S + o_pairs);
@@ -257,6 +258,7 @@ extern "C" int kvdro_eval_grid_noalloc(int32_t K, const int64_t* offsets, const 
     a.L = mt.L;
     a.L_in = mt.L_in;
     a.cdf = sa.hist;
+    a.csum = nullptr;
     a.hist_off = sa.hist_off;
     a.r = reinterpret_cast<const int32_t*>(S + o_r);
     a.lam = reinterpret_cast<const double*>(S + o_lam);

@@ -72,13 +72,64 @@ __global__ void __launch_bounds__(kHistThreads) k_histogram(SortArgs a) {
     }
 }
 
-// In-place inclusive scan of one class's histogram per block.
+// Block-wide inclusive scan of one value per thread; returns the thread's inclusive prefix and
+// leaves the block total in *total (all threads).
+template <typename T>
+__device__ __forceinline__ T block_inclusive_scan(T t, T* warp_tot, T* total) {
+    const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+    T incl = t;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const T y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (l >= o) incl += y;
+    }
+    if (l == 31) warp_tot[w] = incl;
+    __syncthreads();
+    if (w == 0) {
+        T s = warp_tot[l];
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const T y = __shfl_up_sync(0xffffffffu, s, o);
+            if (l >= o) s += y;
+        }
+        warp_tot[l] = s;
+    }
+    __syncthreads();
+    const T before = (w ? warp_tot[w - 1] : (T)0) + incl;
+    *total = warp_tot[kScanThreads / 32 - 1];
+    __syncthreads();
+    return before;
+}
+
+// Per class (one block): cumulative sums sum_{x <= v} x (if requested), then the in-place
+// inclusive scan of the histogram into cumulative counts.
 __global__ void __launch_bounds__(kScanThreads) k_scan(SortArgs a) {
     __shared__ int32_t warp_tot[kScanThreads / 32];
+    __shared__ long long warp_tot64[kScanThreads / 32];
     const int k = blockIdx.x;
     int32_t* h = a.hist + a.hist_off[k];
     const int64_t n = (int64_t)a.L[k] + 1;
     const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+    if (a.csum) {
+        long long* cs = reinterpret_cast<long long*>(a.csum + a.hist_off[k]);
+        long long carry64 = 0;
+        for (int64_t base = 0; base < n; base += (int64_t)kScanThreads * 4) {
+            const int64_t i0 = base + (int64_t)threadIdx.x * 4;
+            long long v[4], t = 0;
+#pragma unroll
+            for (int j = 0; j < 4; j++) {
+                v[j] = (i0 + j < n) ? (long long)(i0 + j) * h[i0 + j] : 0;
+                t += v[j];
+                v[j] = t;
+            }
+            long long total;
+            const long long incl = block_inclusive_scan<long long>(t, warp_tot64, &total);
+#pragma unroll
+            for (int j = 0; j < 4; j++)
+                if (i0 + j < n) cs[i0 + j] = carry64 + incl - t + v[j];
+            carry64 += total;
+        }
+    }
     int32_t carry = 0;
     for (int64_t base = 0; base < n; base += (int64_t)kScanThreads * 4) {
         const int64_t i0 = base + (int64_t)threadIdx.x * 4;

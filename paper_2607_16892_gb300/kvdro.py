@@ -32,13 +32,14 @@ KVDRO_ETIMEOUT = -5
 KVDRO_FP32 = 0
 KVDRO_FP64 = 1
 KVDRO_EXACT = 2
+KVDRO_ENVELOPE = 3
 
 _STATUS = {0: "KVDRO_OK", -1: "KVDRO_EINVAL", -2: "KVDRO_ENOMEM", -3: "KVDRO_ECUDA", -4: "KVDRO_ESTATE",
            -5: "KVDRO_ETIMEOUT"}
 
 # Every entry point declared in include/kvdro.h.
 SYMBOLS = ("kvdro_create", "kvdro_load_samples", "kvdro_quantiles", "kvdro_eval_grid", "kvdro_sorted_samples",
-           "kvdro_last_grid_ms", "kvdro_eval_grid_noalloc", "kvdro_sync", "kvdro_last_error", "kvdro_destroy")
+           "kvdro_eval_dual", "kvdro_last_grid_ms", "kvdro_eval_grid_noalloc", "kvdro_sync", "kvdro_last_error", "kvdro_destroy")
 
 _lock = threading.Lock()
 _lib = None
@@ -75,6 +76,8 @@ def load_library(build_if_missing: bool = True) -> ctypes.CDLL:
         lib.kvdro_quantiles.argtypes = [P, i32, P, P, P]
         lib.kvdro_eval_grid.restype = ctypes.c_int
         lib.kvdro_eval_grid.argtypes = [P, ctypes.c_int, i32, P, i32, P, i32, P, i32, P, P, P, P, P, P, P, P, P]
+        lib.kvdro_eval_dual.restype = ctypes.c_int
+        lib.kvdro_eval_dual.argtypes = [P, i32, P, i32, P, i32, P, P, P, P, P, P, P, P]
         lib.kvdro_sorted_samples.restype = ctypes.c_int
         lib.kvdro_sorted_samples.argtypes = [P, P, P]
         lib.kvdro_last_grid_ms.restype = ctypes.c_int
@@ -175,6 +178,16 @@ def kvdro_eval_grid(ctx, precision: int, R: int, r, NL: int, lam, E: int, eps, M
         ctx, int(precision), int(R), rr.ctypes.data, int(NL), ll.ctypes.data, int(E), ee.ctypes.data, int(M),
         cp.ctypes.data, cw.ctypes.data, _ptr(S, ft), _ptr(cost, ft), _ptr(lam_idx, np.int32), _ptr(r_idx, np.int32),
         _ptr(min_cost, ft), _ptr(fhat, np.float64), _stream(stream)))
+
+
+def kvdro_eval_dual(ctx, R: int, r, E: int, eps, M: int, c_p, c_w, cost=None, gamma=None, r_idx=None,
+                    min_cost=None, fhat=None, stream=None) -> None:
+    rr, ee = _host(r, np.int32), _host(eps, np.float64)
+    cp, cw = _host(c_p, np.float64), _host(c_w, np.float64)
+    _check(ctx, load_library().kvdro_eval_dual(
+        ctx, int(R), rr.ctypes.data, int(E), ee.ctypes.data, int(M), cp.ctypes.data, cw.ctypes.data,
+        _ptr(cost, np.float64), _ptr(gamma, np.float64), _ptr(r_idx, np.int32), _ptr(min_cost, np.float64),
+        _ptr(fhat, np.float64), _stream(stream)))
 
 
 def kvdro_sorted_samples(ctx, out, stream=None) -> None:

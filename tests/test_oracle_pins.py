@@ -356,3 +356,40 @@ def test_quantile_rank_convention():
     assert O.quantile_rank(0.951, 20) == 20
     assert O.quantile_rank(1.0 / 3.0, 3) == 1
     assert math.isclose(20.0 / 21.0, O.quantile_rank(20.0 / 21.0, 21) / 21.0)
+
+
+# ----------------------------------------------------------------- the exact dual (no lam grid)
+
+def test_exact_dual_equals_the_paper_lp_and_the_primal_worst_case():
+    rng = np.random.default_rng(14)
+    for _ in range(40):
+        L = int(rng.integers(4, 30))
+        n = int(rng.integers(1, 6))
+        xs = rng.integers(0, L + 1, n)
+        eta = int(rng.integers(0, L + 1))
+        eps = float(rng.choice([0.0, rng.uniform(0, 3), rng.uniform(0, L)]))
+        cp, cw = float(rng.uniform(0.5, 25)), float(rng.uniform(0.2, 4))
+        w = one_class(xs, L, [eta], [1.0], [eps], cp, cw)
+        got = O.solve_dual(w)["cost"][0, 0, 0, 0]
+        lp, _ = _dual_lp(xs, eta, eps, cp, cw, L)
+        assert abs(got - lp) <= 1e-7 * max(1.0, abs(lp))
+        if L <= 20:
+            assert abs(got - _primal_lp(xs, eta, eps, cp, cw, L)) <= 1e-7 * max(1.0, abs(lp))
+
+
+def test_exact_dual_closed_forms_and_grid_bound():
+    w = random_case(15, K=2, N=(400, 23), L=(300, 300), R=13, n_lam=24, n_eps=4, M=2, eps_max=250.0,
+                    lam_range=(1e-3, 300.0))
+    w.eps = np.array([0.0, 3.0, 60.0, 400.0])  # the last radius exceeds L
+    d = O.solve_dual(w)
+    g = O.solve(w)
+    assert np.all(d["cost"] <= g["cost"] * (1 + 1e-12) + 1e-12)        # the grid restricts gamma
+    for m in range(2):
+        for k in range(2):
+            for i, r in enumerate(w.r):
+                eta = int(r - w.L_in[k])
+                saa = survival_saa(w.class_samples(k), eta, w.cp[m], w.cw[m], int(w.L[k]))
+                assert abs(d["cost"][m, 0, k, i] - saa) <= 1e-11 * max(1.0, saa)                # eps = 0
+                worst = max(w.cw[m] * eta, w.cp[m] * (int(w.L[k]) - eta))
+                assert abs(d["cost"][m, 3, k, i] - worst) <= 1e-11 * max(1.0, worst)           # eps >= L
+    assert np.all(np.diff(d["cost"], axis=1) >= -1e-9)                                        # monotone in eps
