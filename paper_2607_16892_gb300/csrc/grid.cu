@@ -33,8 +33,6 @@ namespace {
 
 typedef unsigned long long u64;
 
-constexpr int kChunk = 2048;      // samples per staged chunk (16 KB of float2)
-constexpr int kStages = 3;        // ring depth
 constexpr long long kWaitCycles = 4000000000LL;  // ~2 s at 2 GHz: bound on any barrier wait
 
 constexpr int ilog2(int v) { return v <= 1 ? 0 : 1 + ilog2(v / 2); }
@@ -43,20 +41,27 @@ constexpr int ilog2(int v) { return v <= 1 ? 0 : 1 + ilog2(v / 2); }
 // multipliers, TR*TL a power of two <= 32), FP32 chunks between folds of the per-lane partial
 // sums into FP64 (FP64 folds once at the end), and the largest CTA and minimum CTAs per SM it is
 // compiled for (these two bound its registers per thread).
-template <Prec P_, int TR_, int TL_, int FLUSH_, int MINB_, int MAXT_ = 512>
+template <Prec P_, int TR_, int TL_, int FLUSH_, int MINB_, int MAXT_ = 512, int CHUNK_ = 2048, int STAGES_ = 3,
+          int UNROLL_ = 2>
 struct GridCfg {
     static constexpr Prec P = P_;
     static constexpr int TR = TR_, TL = TL_, V = TR_ * TL_, LOG2V = ilog2(TR_ * TL_), FLUSH = FLUSH_, MINB = MINB_;
     static constexpr int MAXT = MAXT_;
+    static constexpr int CHUNK = CHUNK_;    // samples per staged chunk (float2 each)
+    static constexpr int STAGES = STAGES_;  // ring depth
+    static constexpr int UNROLL = UNROLL_;  // unroll of the FP32 sample loop
+    static_assert(CHUNK_ % 128 == 0 && CHUNK_ * 8 * STAGES_ <= 160 * 1024, "chunk ring must fit shared memory");
     static_assert((V & (V - 1)) == 0 && V >= 2 && V <= 32, "tile must hold a power of two <= 32 cells");
     static_assert(P_ == Prec::F64 || TL_ % 2 == 0, "the FP32 and exact tiles pack lam values in pairs");
 };
 // FP32: 2 r x 8 lam tiles, up to 16 warps per CTA and two CTAs per SM (64 registers) for up to
 // 128 lam values; 2 x 16 tiles for 129..256 lam values.  FP64: 2 x 8 tiles.
-using CfgF32 = GridCfg<Prec::F32, 2, 8, 4, 2, 512>;
-using CfgF32Wide = GridCfg<Prec::F32, 2, 16, 4, 1, 512>;
-using CfgF64 = GridCfg<Prec::F64, 2, 8, 0, 1, 512>;
-using CfgExact = GridCfg<Prec::EXACT, 2, 8, 0, 2, 512>;
+// All stage 4096-sample chunks (32 KB) through a 2-deep ring; the FP32 variants fold their
+// partial sums every 2 chunks (256 samples per lane) and unroll the sample loop 8 times.
+using CfgF32 = GridCfg<Prec::F32, 2, 8, 2, 2, 512, 4096, 2, 8>;
+using CfgF32Wide = GridCfg<Prec::F32, 2, 16, 2, 1, 512, 4096, 2, 2>;
+using CfgF64 = GridCfg<Prec::F64, 2, 8, 0, 1, 512, 4096, 2>;
+using CfgExact = GridCfg<Prec::EXACT, 2, 8, 0, 2, 512, 4096, 2>;
 constexpr int kWarpsTarget = 16;  // warps per CTA the r groups fill up to
 
 // ---------------------------------------------------------------- PTX helpers
@@ -188,11 +193,11 @@ struct SmemLayout {
     size_t ring, full, lam, eps, S, total;
 };
 
-__host__ __device__ inline SmemLayout smem_layout(int RG, int TR, int NLpad, int E) {
+__host__ __device__ inline SmemLayout smem_layout(int RG, int TR, int NLpad, int E, int chunk, int stages) {
     SmemLayout L;
     L.ring = 0;
-    L.full = (size_t)kStages * kChunk * sizeof(float2);
-    L.lam = L.full + 8 * kStages;
+    L.full = (size_t)stages * chunk * sizeof(float2);
+    L.lam = L.full + 8 * (size_t)stages;
     L.eps = L.lam + 8 * (size_t)NLpad;
     L.S = L.eps + 8 * (size_t)E;
     L.total = L.S + 8 * (size_t)RG * TR * NLpad;
@@ -249,14 +254,14 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
     constexpr int TR = C::TR, TL = C::TL, V = C::V, LOG2V = C::LOG2V;
     extern __shared__ __align__(128) unsigned char smem[];
     const int NLpad = a.LT * TL;
-    const SmemLayout lay = smem_layout(a.RG, TR, NLpad, a.E);
+    const SmemLayout lay = smem_layout(a.RG, TR, NLpad, a.E, C::CHUNK, C::STAGES);
     float2* ring = reinterpret_cast<float2*>(smem + lay.ring);
     u64* full = reinterpret_cast<u64*>(smem + lay.full);
     double* s_lam = reinterpret_cast<double*>(smem + lay.lam);
     double* s_eps = reinterpret_cast<double*>(smem + lay.eps);
     double* s_S = reinterpret_cast<double*>(smem + lay.S);
 
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nwarps = blockDim.x >> 5;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     int b = blockIdx.x;
     const int rb = b % a.r_blocks;
     b /= a.r_blocks;
@@ -271,22 +276,22 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
 
     const int64_t pbase = a.pair_off[k];
     const int64_t np = a.pair_off[k + 1] - pbase;  // multiple of kPadSamples
-    const int nchunks = (int)((np + kChunk - 1) / kChunk);
+    const int nchunks = (int)((np + C::CHUNK - 1) / C::CHUNK);
     const float2* src = a.pairs + pbase;
     auto issue = [&](int c) {
-        const int s = c % kStages;
-        const int64_t cnt = min((int64_t)kChunk, np - (int64_t)c * kChunk);
-        tma_bulk_load(smem_u32(ring + (size_t)s * kChunk), src + (int64_t)c * kChunk, (uint32_t)(cnt * sizeof(float2)),
+        const int s = c % C::STAGES;
+        const int64_t cnt = min((int64_t)C::CHUNK, np - (int64_t)c * C::CHUNK);
+        tma_bulk_load(smem_u32(ring + (size_t)s * C::CHUNK), src + (int64_t)c * C::CHUNK, (uint32_t)(cnt * sizeof(float2)),
                       smem_u32(&full[s]));
     };
     if (tid == 0) {
-        for (int s = 0; s < kStages; s++) mbar_init(smem_u32(&full[s]), 1);
+        for (int s = 0; s < C::STAGES; s++) mbar_init(smem_u32(&full[s]), 1);
         fence_mbar_init();
     }
     __syncthreads();
     if (tid == 0)
-        for (int c = 0; c < kStages && c < nchunks; c++) issue(c);
-    int issued = min(kStages, nchunks);  // chunks issued so far (tracked identically by every thread)
+        for (int c = 0; c < C::STAGES && c < nchunks; c++) issue(c);
+    int issued = min(C::STAGES, nchunks);  // chunks issued so far (tracked identically by every thread)
     int consumed = 0;                    // chunk at which the loop stopped
 
     // Per-cell constants of this warp's tile (identical across its lanes).
@@ -321,13 +326,13 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
             }
         }
         for (int c = 0; c < nchunks; c++) {
-            const int s = c % kStages;
-            if (!mbar_wait_bounded(smem_u32(&full[s]), (uint32_t)((c / kStages) & 1))) timeout = true;
+            const int s = c % C::STAGES;
+            if (!mbar_wait_bounded(smem_u32(&full[s]), (uint32_t)((c / C::STAGES) & 1))) timeout = true;
             if (!timeout) {
-                const int cnt = (int)min((int64_t)kChunk, np - (int64_t)c * kChunk);
-                const float4* q = reinterpret_cast<const float4*>(ring + (size_t)s * kChunk);
+                const int cnt = (int)min((int64_t)C::CHUNK, np - (int64_t)c * C::CHUNK);
+                const float4* q = reinterpret_cast<const float4*>(ring + (size_t)s * C::CHUNK);
                 const int nq = cnt >> 6;  // float4 (two samples) per lane
-#pragma unroll 2
+#pragma unroll(C::UNROLL)
                 for (int t = 0; t < nq; t++) {
                     const float4 v = q[lane + 32 * t];
                     const u64 xa = pk(v.x, v.y), xb = pk(v.z, v.w);
@@ -362,12 +367,12 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
                 timeout = true;
                 break;
             }
-            if (c + kStages < nchunks) {
+            if (c + C::STAGES < nchunks) {
                 if (tid == 0) {
                     fence_proxy_async();
-                    issue(c + kStages);
+                    issue(c + C::STAGES);
                 }
-                issued = c + kStages + 1;
+                issued = c + C::STAGES + 1;
             }
         }
     } else if constexpr (P == Prec::F64) {
@@ -386,11 +391,11 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
             }
         }
         for (int c = 0; c < nchunks; c++) {
-            const int s = c % kStages;
-            if (!mbar_wait_bounded(smem_u32(&full[s]), (uint32_t)((c / kStages) & 1))) timeout = true;
+            const int s = c % C::STAGES;
+            if (!mbar_wait_bounded(smem_u32(&full[s]), (uint32_t)((c / C::STAGES) & 1))) timeout = true;
             if (!timeout) {
-                const int cnt = (int)min((int64_t)kChunk, np - (int64_t)c * kChunk);
-                const float4* q = reinterpret_cast<const float4*>(ring + (size_t)s * kChunk);
+                const int cnt = (int)min((int64_t)C::CHUNK, np - (int64_t)c * C::CHUNK);
+                const float4* q = reinterpret_cast<const float4*>(ring + (size_t)s * C::CHUNK);
                 const int nq = cnt >> 6;
                 for (int t = 0; t < nq; t++) {
                     const float4 v = q[lane + 32 * t];
@@ -409,12 +414,12 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
                 timeout = true;
                 break;
             }
-            if (c + kStages < nchunks) {
+            if (c + C::STAGES < nchunks) {
                 if (tid == 0) {
                     fence_proxy_async();
-                    issue(c + kStages);
+                    issue(c + C::STAGES);
                 }
-                issued = c + kStages + 1;
+                issued = c + C::STAGES + 1;
             }
         }
         if (!timeout) {
@@ -472,11 +477,11 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
         };
         int pending = 0;  // loads since the last fold
         for (int c = 0; c < nchunks; c++) {
-            const int s = c % kStages;
-            if (!mbar_wait_bounded(smem_u32(&full[s]), (uint32_t)((c / kStages) & 1))) timeout = true;
+            const int s = c % C::STAGES;
+            if (!mbar_wait_bounded(smem_u32(&full[s]), (uint32_t)((c / C::STAGES) & 1))) timeout = true;
             if (!timeout) {
-                const int cnt = (int)min((int64_t)kChunk, np - (int64_t)c * kChunk);
-                const float4* q = reinterpret_cast<const float4*>(ring + (size_t)s * kChunk);
+                const int cnt = (int)min((int64_t)C::CHUNK, np - (int64_t)c * C::CHUNK);
+                const float4* q = reinterpret_cast<const float4*>(ring + (size_t)s * C::CHUNK);
                 const int nq = cnt >> 6;
                 for (int t0 = 0; t0 < nq; t0 += fe) {
                     const int t1 = min(nq, t0 + fe);
@@ -509,12 +514,12 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
                 timeout = true;
                 break;
             }
-            if (c + kStages < nchunks) {
+            if (c + C::STAGES < nchunks) {
                 if (tid == 0) {
                     fence_proxy_async();
-                    issue(c + kStages);
+                    issue(c + C::STAGES);
                 }
-                issued = c + kStages + 1;
+                issued = c + C::STAGES + 1;
             }
         }
         if (!timeout) {
@@ -535,7 +540,7 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
         if (tid == 0) {
             atomicOr(a.err + 1, kErrTimeout);
             for (int c = consumed; c < issued; c++)
-                (void)mbar_wait_bounded(smem_u32(&full[c % kStages]), (uint32_t)((c / kStages) & 1));
+                (void)mbar_wait_bounded(smem_u32(&full[c % C::STAGES]), (uint32_t)((c / C::STAGES) & 1));
         }
         __syncthreads();
         return;
@@ -652,7 +657,7 @@ GridShape shape_for(int variant, int32_t R, int32_t NL, int32_t E) {
     sh.RG = sh.LT >= kWarpsTarget ? 1 : kWarpsTarget / sh.LT;
     sh.threads = 32 * sh.LT * sh.RG;
     sh.r_blocks = (R + sh.RG * C::TR - 1) / (sh.RG * C::TR);
-    sh.smem = smem_layout(sh.RG, C::TR, sh.LT * C::TL, E).total;
+    sh.smem = smem_layout(sh.RG, C::TR, sh.LT * C::TL, E, C::CHUNK, C::STAGES).total;
     return sh;
 }
 
@@ -675,7 +680,7 @@ GridShape grid_shape(Prec p, int32_t R, int32_t NL, int32_t E) {
 
 cudaError_t grid_prepare(Prec p) {
     // the largest layout any variant can need: 16 warps, 256 lam, 64 eps
-    const int mx = (int)(smem_layout(16, 2, 256, 64).total + 4096);
+    const int mx = (int)(smem_layout(16, 2, 256, 64, 4096, 4).total + 4096);
     if (p == Prec::F64) return cudaFuncSetAttribute(k_grid<CfgF64>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
     if (p == Prec::EXACT) return cudaFuncSetAttribute(k_grid<CfgExact>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
     if (p == Prec::ENVELOPE)
