@@ -63,6 +63,9 @@ def parse_args():
     p.add_argument("--cpu-seconds", type=float, default=10.0, help="target wall time of the CPU-baseline sample")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--drift-iterations", type=int, default=3)
+    p.add_argument("--case", default="",
+                   help="WORKLOAD:MODE, MODE in fp32|fp64|exact|envelope|dual|sort: time one kernel path "
+                        "(--warmup untimed, --steps timed runs) and print one line per run")
     p.add_argument("--suite", action="store_true",
                    help="time every workload in each precision (one JSON line per case) instead of the contract line")
     return p.parse_args()
@@ -424,8 +427,41 @@ def run_suite(args):
                                                                 "terms_per_s")}}), flush=True)
 
 
+def run_case(args):
+    """One workload through one path, for profiling: load + sort, then the chosen evaluation."""
+    import torch
+
+    from paper_2607_16892_gb300 import kvdro as kv
+    from synth import WORKLOADS
+
+    name, mode = args.case.split(":")
+    w = WORKLOADS[name]()
+    dev = torch.device("cuda", 0)
+    M, E, K, R, NL = len(w.cp), len(w.eps), w.K, len(w.r), len(w.lam)
+    ctx = kv.kvdro_create(0)
+    d = torch.from_numpy(w.samples).to(dev)
+    r_idx = torch.empty((M, E, K), dtype=torch.int32, device=dev)
+    prec = {"fp32": kv.KVDRO_FP32, "fp64": kv.KVDRO_FP64, "exact": kv.KVDRO_EXACT, "envelope": kv.KVDRO_ENVELOPE}
+    for i in range(args.warmup + args.steps):
+        t0 = time.perf_counter()
+        kv.kvdro_load_samples(ctx, K, w.offsets, d, w.L, w.L_in)
+        if mode == "dual":
+            kv.kvdro_eval_dual(ctx, R, w.r, E, w.eps, M, w.cp, w.cw, r_idx=r_idx)
+        elif mode != "sort":
+            kv.kvdro_eval_grid(ctx, prec[mode], R, w.r, NL, w.lam, E, w.eps, M, w.cp, w.cw, r_idx=r_idx)
+        torch.cuda.synchronize(dev)
+        line = {"case": args.case, "run": i, "timed": i >= args.warmup, "wall_ms": 1e3 * (time.perf_counter() - t0)}
+        if mode != "sort":
+            line["kernel_ms"] = kv.kvdro_last_grid_ms(ctx)
+        print(json.dumps(line), flush=True)
+    kv.kvdro_destroy(ctx)
+
+
 def main():
     args = parse_args()
+    if args.case:
+        run_case(args)
+        return
     if args.suite:
         run_suite(args)
         return

@@ -12,6 +12,8 @@
 #include <string>
 #include <vector>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "kvdro.h"
 #include "kvdro_internal.cuh"
 
@@ -89,6 +91,12 @@ int cuda_fail(kvdro_ctx* c, cudaError_t e, const char* what) {
         cudaError_t e_ = (call);                       \
         if (e_ != cudaSuccess) return cuda_fail(ctx, e_, what); \
     } while (0)
+
+// An NVTX range around one entry point (visible in Nsight timelines; a no-op without a tool).
+struct NvtxRange {
+    explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+    ~NvtxRange() { nvtxRangePop(); }
+};
 
 // Keeps the caller's current device and restores it on exit.
 struct DeviceGuard {
@@ -240,6 +248,7 @@ const char* kvdro_last_error(const kvdro_ctx* ctx) { return ctx ? ctx->err.c_str
 
 int kvdro_load_samples(kvdro_ctx* ctx, int32_t K, const int64_t* offsets, const int32_t* lengths,
                        const int32_t* L_max, const int32_t* L_in, void* stream) {
+    NvtxRange nvtx_("kvdro_load_samples");
     if (!ctx) return KVDRO_EINVAL;
     ctx->err.clear();
     if (K < 1 || K > kMaxK) return fail(ctx, KVDRO_EINVAL, "K = %d outside [1, %d]", K, kMaxK);
@@ -359,6 +368,7 @@ int kvdro_load_samples(kvdro_ctx* ctx, int32_t K, const int64_t* offsets, const 
 }
 
 int kvdro_quantiles(kvdro_ctx* ctx, int32_t F, const double* fractiles, int32_t* out, void* stream) {
+    NvtxRange nvtx_("kvdro_quantiles");
     if (!ctx) return KVDRO_EINVAL;
     ctx->err.clear();
     if (!ctx->loaded) return fail(ctx, KVDRO_ESTATE, "no samples loaded");
@@ -407,6 +417,7 @@ int kvdro_quantiles(kvdro_ctx* ctx, int32_t F, const double* fractiles, int32_t*
 int kvdro_eval_grid(kvdro_ctx* ctx, int precision, int32_t R, const int32_t* r, int32_t NL, const double* lam,
                     int32_t E, const double* eps, int32_t M, const double* c_p, const double* c_w, void* S,
                     void* cost, int32_t* lam_idx, int32_t* r_idx, void* min_cost, double* fhat, void* stream) {
+    NvtxRange nvtx_("kvdro_eval_grid");
     if (!ctx) return KVDRO_EINVAL;
     ctx->err.clear();
     if (!ctx->loaded) return fail(ctx, KVDRO_ESTATE, "no samples loaded");
@@ -571,6 +582,7 @@ int kvdro_eval_grid(kvdro_ctx* ctx, int precision, int32_t R, const int32_t* r, 
 int kvdro_eval_dual(kvdro_ctx* ctx, int32_t R, const int32_t* r, int32_t E, const double* eps, int32_t M,
                     const double* c_p, const double* c_w, double* cost, double* gamma, int32_t* r_idx,
                     double* min_cost, double* fhat, void* stream) {
+    NvtxRange nvtx_("kvdro_eval_dual");
     if (!ctx) return KVDRO_EINVAL;
     ctx->err.clear();
     if (!ctx->loaded) return fail(ctx, KVDRO_ESTATE, "no samples loaded");
@@ -699,6 +711,7 @@ int kvdro_eval_dual(kvdro_ctx* ctx, int32_t R, const int32_t* r, int32_t E, cons
 }
 
 int kvdro_sorted_samples(const kvdro_ctx* cctx, int32_t* out, void* stream) {
+    NvtxRange nvtx_("kvdro_sorted_samples");
     kvdro_ctx* ctx = const_cast<kvdro_ctx*>(cctx);
     if (!ctx) return KVDRO_EINVAL;
     ctx->err.clear();
@@ -728,6 +741,7 @@ int kvdro_last_grid_ms(kvdro_ctx* ctx, float* ms) {
 }
 
 int kvdro_sync(kvdro_ctx* ctx) {
+    NvtxRange nvtx_("kvdro_sync");
     if (!ctx) return KVDRO_EINVAL;
     ctx->err.clear();
     DeviceGuard g(ctx->device);

@@ -11,6 +11,8 @@
 #include <initializer_list>
 #include <mutex>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "kvdro.h"
 #include "kvdro_internal.cuh"
 
@@ -108,6 +110,8 @@ extern "C" int kvdro_eval_grid_noalloc(int32_t K, const int64_t* offsets, const 
                                        const double* c_p, const double* c_w, float* cost, int32_t* lam_idx,
                                        int32_t* r_idx, float* min_cost, double* fhat, void* stream, char* err,
                                        int32_t err_len) {
+    nvtxRangePushA("kvdro_eval_grid_noalloc");
+    struct PopAtExit { ~PopAtExit() { nvtxRangePop(); } } pop_at_exit_;
     if (err && err_len > 0) err[0] = 0;
     // ---- host-side validation (the rules of kvdro_load_samples and of kvdro_eval_grid in FP32)
     if (K < 1 || K > 4096) return report(err, err_len, KVDRO_EINVAL, "K outside [1, 4096]");

@@ -17,7 +17,7 @@ from __future__ import annotations
 import ctypes
 import os
 import threading
-from typing import Any, Optional
+from typing import Any
 
 import numpy as np
 
@@ -96,9 +96,6 @@ def load_library(build_if_missing: bool = True) -> ctypes.CDLL:
 
 
 # ------------------------------------------------------------------ marshalling
-
-_keep: list = []
-
 
 def _ptr(a: Any, dtype=None):
     """Pointer to the data of a NumPy array or torch tensor (None -> NULL)."""
