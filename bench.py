@@ -68,6 +68,8 @@ def parse_args():
                         "(--warmup untimed, --steps timed runs) and print one line per run")
     p.add_argument("--suite", action="store_true",
                    help="time every workload in each precision (one JSON line per case) instead of the contract line")
+    p.add_argument("--bcd", action="store_true",
+                   help="time the block-coordinate descent (Alg. 1) on the scalability instances, one line each")
     return p.parse_args()
 
 
@@ -436,6 +438,38 @@ def run_suite(args):
                                                                 "terms_per_s")}}), flush=True)
 
 
+# BCD-DRO solve times of the paper's scalability table (Sec. 5.2; hardware unstated), by
+# (classes, configurations, samples per class): context for the host solve, not a target
+PAPER_BCD_SECONDS = {(3, 4, 100): 0.17, (4, 4, 150): 0.8, (5, 5, 200): 4.3, (6, 6, 300): 10.5, (8, 6, 500): 22.4,
+                     (10, 8, 1000): 81.2, (15, 12, 2000): 257.7}
+
+
+def run_bcd(args):
+    """Alg. 1 end to end on the scalability instances: the library's worst-case cost tables
+    (one exact-dual pass per support size) and the host blocks, each timed on the wall clock."""
+    from paper_2607_16892_gb300 import bcd
+    from synth import SCALABILITY_SIZES, bcd_instance
+
+    warm = bcd.Problem(**bcd_instance(2, 2, 50, 8, L_cap=64))
+    bcd.solve(warm, bcd.gpu_tables(warm))          # library load, CUDA context, scipy import
+    for I, K, N, J in SCALABILITY_SIZES:
+        p = bcd.Problem(**bcd_instance(I, K, N, J))
+        t0 = time.perf_counter()
+        tables = bcd.gpu_tables(p)
+        res = bcd.solve(p, tables)
+        total = time.perf_counter() - t0
+        sec = res.seconds
+        print(json.dumps({"bcd": True, "instance": p.name, "classes": I, "configs": K, "samples_per_class": N,
+                          "gpus_modelled": J, "configurations_in_Z": int(bcd.config_set(p.tau * p.pp, p.J).shape[0]),
+                          "total_s": total, "tables_s": sec["tables"], "lp1_s": sec["lp1"], "lp2_s": sec["lp2"],
+                          "block3_s": sec["block3"], "lp_rounds": res.lp_rounds,
+                          "outer_iterations": res.outer_iterations, "objective": res.objective,
+                          "admitted": float((p.arrival * res.pi.sum(axis=1)).sum() / p.arrival.sum()),
+                          "paper_bcd_s": PAPER_BCD_SECONDS.get((I, K, N)),
+                          "paper_note": "paper's BCD-DRO time, hardware unstated, LP over per-sample epigraph "
+                                        "variables; context only"}), flush=True)
+
+
 def run_case(args):
     """One workload through one path, for profiling: load + sort, then the chosen evaluation."""
     import torch
@@ -471,8 +505,12 @@ def main():
     if args.case:
         run_case(args)
         return
+    if args.bcd:
+        run_bcd(args)
+        return
     if args.suite:
         run_suite(args)
+        run_bcd(args)
         return
     if args.impl == "reference":
         run_reference(args)

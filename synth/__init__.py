@@ -16,3 +16,4 @@ from .workloads import (  # noqa: F401
     random_case,
     slice_workload,
 )
+from .bcd_instances import CONFIGS, SCALABILITY_SIZES, bcd_instance  # noqa: F401
