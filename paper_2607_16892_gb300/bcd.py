@@ -164,21 +164,20 @@ def service_cv2(p: Problem) -> np.ndarray:
 
 
 def config_set(gpus_per_group: np.ndarray, J: int) -> np.ndarray:
-    """Every z in Z_+^nK with sum_k z_k g_k <= J, in lexicographic order (Sec. 4.3)."""
-    g = [int(v) for v in gpus_per_group]
-    rows: List[List[int]] = []
-
-    def rec(k: int, left: int, prefix: List[int]):
-        if k == len(g):
-            rows.append(list(prefix))
-            return
-        for zk in range(left // g[k] + 1):
-            prefix.append(zk)
-            rec(k + 1, left - zk * g[k], prefix)
-            prefix.pop()
-
-    rec(0, int(J), [])
-    return np.asarray(rows, dtype=np.int32).reshape(-1, len(g))
+    """Every z in Z_+^nK with sum_k z_k g_k <= J, in lexicographic order (Sec. 4.3).  Built one
+    configuration at a time: each partial vector is repeated once per count its remaining
+    budget allows, the counts ascending."""
+    g = np.asarray(gpus_per_group, np.int64)
+    rows = np.zeros((1, 0), np.int32)
+    left = np.array([int(J)], np.int64)
+    for gk in g:
+        counts = left // int(gk) + 1
+        rep = np.repeat(np.arange(rows.shape[0]), counts)
+        starts = np.repeat(np.cumsum(counts) - counts, counts)
+        zk = (np.arange(rep.size) - starts).astype(np.int64)
+        rows = np.concatenate([rows[rep], zk[:, None].astype(np.int32)], axis=1)
+        left = left[rep] - zk * int(gk)
+    return rows
 
 
 def waiting_time(p: Problem, T: np.ndarray, cv2: np.ndarray, pi: np.ndarray, z: np.ndarray) -> np.ndarray:
@@ -389,36 +388,44 @@ def block2(p: Problem, T: np.ndarray, z: np.ndarray, pi: np.ndarray) -> np.ndarr
 
 
 def block3(p: Problem, T: np.ndarray, cv2: np.ndarray, Z: np.ndarray, z_cur: np.ndarray, eta: np.ndarray,
-           pi: np.ndarray, delta: np.ndarray, d: np.ndarray, chunk: int = 65536):
+           pi: np.ndarray, delta: np.ndarray, d: np.ndarray, chunk: int = 131072):
     """z = argmin over Z of the objective with (r, pi, delta) fixed (Alg. 1 Block 3), every z
-    evaluated.  Returns (z, its objective); the current z when nothing is feasible."""
-    I, nK = p.I, p.nK
+    evaluated.  With pi fixed, configuration k's feasibility (routing consistency, utilisation,
+    eq. capacity) and waiting time depend on z_k alone, so they are tabulated per (k, z_k) and
+    gathered; the SLO slack of every class is then one product with pi.  Returns (z, its
+    objective); the current z when nothing is feasible."""
     a = pi.sum(axis=1)
     load = (p.arrival[:, None] * pi * T).sum(axis=0)           # U_k
     rate = (p.arrival[:, None] * pi).sum(axis=0)
-    tbar = np.where(rate > 0, load / np.where(rate > 0, rate, 1.0), 0.0)
+    routed = rate > 0
+    tbar = np.where(routed, load / np.where(routed, rate, 1.0), 0.0)
     u_ik = p.arrival[:, None] * T
     r_t = _reservation(p, eta)[:, None] - delta * p.L_pre[:, None]
-    capload = (1.0 + p.kappa) * (u_ik * pi * r_t).sum(axis=0)   # z_k * (capacity LHS minus prefixes)
+    capload = (1.0 + p.kappa) * (u_ik * pi * r_t).sum(axis=0)   # z_k times the capacity term
     prefix = (delta * p.L_pre[:, None]).sum(axis=0)
-    routed = rate > 0
+    zmax = int(Z.max()) if Z.size else 0
+    ok_t = np.zeros((p.nK, zmax + 1), bool)
+    W_t = np.zeros((p.nK, zmax + 1))
+    for k in range(p.nK):
+        ok_t[k, 0] = not routed[k]
+        for v in range(1, zmax + 1):
+            u = load[k] / v
+            ok = u <= p.u_max * (1 + 1e-9) and u < 1.0
+            ok = ok and capload[k] / v + prefix[k] - p.M[k] <= 1e-7 * max(p.M[k], 1.0)
+            ok_t[k, v] = ok
+            if ok and routed[k]:
+                W_t[k, v] = u * (1.0 + cv2[k]) / (2.0 * (1.0 - u)) * tbar[k]
+    base = (pi * T).sum(axis=1) - a * p.D                     # [I]
+    wslo = p.arrival * p.c_slo
     gpu = (pi * p.c_gpu * (p.tau * p.pp)[None, :] * T).sum(axis=1)
     const = float((p.arrival * (a * d + gpu + (1.0 - a) * p.c_rej)).sum())
-    best_val, best_idx = np.inf, -1
+    kk = np.arange(p.nK)[None, :]
     vals_all = np.empty(Z.shape[0])
     for s0 in range(0, Z.shape[0], chunk):
-        zc = Z[s0:s0 + chunk].astype(np.float64)               # [n, nK]
-        ok = ~np.any(routed[None, :] & (zc <= 0), axis=1)
-        zs = np.where(zc > 0, zc, 1.0)
-        u = np.where(zc > 0, load[None, :] / zs, 0.0)
-        ok &= np.all(u <= p.u_max * (1 + 1e-9), axis=1) & np.all(u < 1.0, axis=1)
-        cap = np.where(zc > 0, capload[None, :] / zs + prefix[None, :] - p.M[None, :], -1.0)
-        ok &= np.all(cap <= 1e-7 * np.maximum(p.M, 1.0)[None, :], axis=1)
-        with np.errstate(divide="ignore", invalid="ignore"):
-            W = np.where(routed[None, :] & (zc > 0), u * (1.0 + cv2[None, :]) / (2.0 * (1.0 - u)) * tbar[None, :], 0.0)
-        lat = (pi[None, :, :] * (W[:, None, :] + T[None, :, :])).sum(axis=2)     # [n, I]
-        s = np.maximum(lat - (a * p.D)[None, :], 0.0)
-        val = const + (s * (p.arrival * p.c_slo)[None, :]).sum(axis=1)
+        zc = Z[s0:s0 + chunk]
+        ok = np.all(ok_t[kk, zc], axis=1)
+        lat = W_t[kk, zc] @ pi.T + base[None, :]               # [n, I]
+        val = const + np.maximum(lat, 0.0) @ wslo
         val[~ok] = np.inf
         vals_all[s0:s0 + chunk] = val
     best_idx = int(np.argmin(vals_all))
@@ -453,7 +460,8 @@ def initial_z(p: Problem) -> np.ndarray:
 
 
 def solve(p: Problem, tables: Tables, T_max: int = 20, inner_max: int = 100, steps: int = 7,
-          tol: float = 1e-9, Z: Optional[np.ndarray] = None, log=None) -> BcdResult:
+          tol: float = 1e-9, Z: Optional[np.ndarray] = None, z0: Optional[np.ndarray] = None,
+          log=None) -> BcdResult:
     """Alg. 1: Block 1 (LP1 / LP2 alternation), Block 2, Block 3, until (z, delta) repeats.
 
     LP1 holds the waiting times at those of the current routing; its solution pi' is taken
@@ -462,7 +470,8 @@ def solve(p: Problem, tables: Tables, T_max: int = 20, inner_max: int = 100, ste
     objective of eq. dro_obj, then LP2 re-optimises r exactly.  Block 1 ends when a round
     lowers the objective by less than ``tol`` (relative) or after ``inner_max`` rounds.
     Block 3 keeps z unless another z is strictly better, so no block update raises the
-    objective (the premise of Prop. "Convergence")."""
+    objective (the premise of Prop. "Convergence").  ``z0`` replaces the default first
+    deployment (a warm start from the deployment in service)."""
     t_all = time.perf_counter()
     secs = {"tables": tables.seconds, "lp1": 0.0, "lp2": 0.0, "block2": 0.0, "block3": 0.0}
     T = service_time(p)
@@ -471,7 +480,9 @@ def solve(p: Problem, tables: Tables, T_max: int = 20, inner_max: int = 100, ste
     if Z is None:
         Z = config_set(p.tau * p.pp, p.J)
     secs["enumerate_Z"] = time.perf_counter() - t0
-    z = initial_z(p)
+    z = initial_z(p) if z0 is None else np.asarray(z0, np.int32).copy()
+    if int((z * p.tau * p.pp).sum()) > p.J or np.any(z < 0):
+        raise ValueError("z0 is outside the configuration set")
     delta = np.zeros((p.I, p.nK), np.int32)
     eta = tables.eta0.astype(np.int64).copy()
     d = tables.d0.copy()              # gamma^(0) eps + S(eta^(0), gamma^(0)) until the first LP2

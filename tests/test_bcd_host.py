@@ -315,3 +315,22 @@ def test_solve_at_eps0_reserves_the_critical_fractile():
             x = np.sort(p.class_samples(i))
             assert res.eta[i] == x[O.quantile_rank(q, x.size) - 1]
     assert res.pi.sum() > 0
+
+
+def test_block3_hands_an_unusable_configuration_to_a_routed_one():
+    """A configuration with no KV capacity can carry no traffic (eq. capacity); starting from a
+    deployment that holds two of its groups, Block 3 moves those GPUs to the routed
+    configuration (fewer waits, eq. waiting_time), and the next Block 1 admits more."""
+    p = small_problem(I=4, K=4, N=150, J=8, L_cap=512, load=0.9)
+    p.M = p.M.copy()
+    p.M[0] = 0.0
+    tb = oracle_tables(p)
+    res = bcd.solve(p, tb, z0=np.array([2, 1, 0, 0]))
+    assert res.history[0]["z"] == [0, 2, 0, 0]
+    assert res.outer_iterations >= 2
+    assert np.all(res.pi[:, 0] == 0.0)
+    assert res.history[1]["objective"] < res.history[0]["objective"]
+    tr = np.asarray(res.trace)
+    assert np.all(tr[1:] <= tr[:-1] * (1 + 1e-12) + 1e-12)
+    with pytest.raises(ValueError):
+        bcd.solve(p, tb, z0=np.array([5, 0, 0, 0]))
