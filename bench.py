@@ -39,14 +39,17 @@ from synth import lognormal_workload_k8_n1e5, slice_workload  # noqa: E402
 METRIC = "DRO cost terms/sec (class×r×λ×sample) on 1 GB300; % of FP32/HBM roofline"
 UNIT = "terms/s"
 SM_MAX_MHZ_RECIPE = 2070.0
-# FP32 lane-operation bound of the grid kernel: every term costs three FP32 lane-operations (one
-# fused multiply-add, one max, one add), and an SM dispatches at most 4 schedulers x 32 lanes =
-# 128 FP32 lane-operations per clock (a packed f32x2 instruction occupies two dispatch cycles).
+# FP32-lane bound of the per-term work: every term needs at least two FP32 lane-operations -- the
+# add (or multiply-add) that forms its excess and the add into the running sum -- and an SM has
+# 128 FP32 lanes, so at most 64 terms per clock per SM.  The remaining operation of a term, the
+# max with zero, runs on the ALU pipe or rides on the add as an absolute value (exact kernel);
+# instruction issue (one per scheduler per clock, two instructions per 32 terms) gives the same
+# 64.  Measured on this GB300: packed f32x2 adds alone reach 127.9 FP32 lane-ops/clk/SM.
 LANE_OPS_PER_CLK_PER_SM = 128.0
-LANE_OPS_PER_TERM = 3.0
+LANE_OPS_PER_TERM = 2.0
 TERMS_PER_CLK_PER_SM = LANE_OPS_PER_CLK_PER_SM / LANE_OPS_PER_TERM
 GRID_SOURCE = os.path.join(ROOT, "paper_2607_16892_gb300", "csrc", "grid.cu")
-PROFILE = os.path.join(ROOT, "profiles", "k_grid_f32_lognormal_k8_n1e5.md")
+PROFILE = os.path.join(ROOT, "profiles", "k_grid_exact_lognormal_k8_n1e5.md")
 LAUNCHES_PER_STEP = 6  # histogram, scan, expand, quantile gather, grid, argmin finalise
 # FP64 pipe bound of the native FP64 mode: per term one DFMA (2.0 per clk per SM) plus one DADD and
 # one max.f64 (1.7 per clk per SM each), measured on this GB300; nominal 1.25 TFLOP/s FP64.
@@ -286,10 +289,10 @@ def run_ours(args):
     achieved = terms / (kernel_ms / 1e3)
     peak = props.multi_processor_count * TERMS_PER_CLK_PER_SM * SM_MAX_MHZ_RECIPE * 1e6
     roofline = {"bound": "alu", "achieved": achieved, "peak": peak, "unit": UNIT, "frac": achieved / peak,
-                "traffic": profile_traffic(), "kernel": "k_grid<F32>",
+                "traffic": profile_traffic(), "kernel": "k_grid<EXACT> (FP32 outputs)",
                 "kernel_ms_mean": kernel_ms,
-                "peak_basis": f"{props.multi_processor_count} SMs x {LANE_OPS_PER_CLK_PER_SM:.0f} FP32 lane-ops/clk/SM "
-                              f"/ {LANE_OPS_PER_TERM:.0f} lane-ops per term x {SM_MAX_MHZ_RECIPE:.0f} MHz"}
+                "peak_basis": f"{props.multi_processor_count} SMs x {LANE_OPS_PER_CLK_PER_SM:.0f} FP32 lanes/clk/SM "
+                              f"/ {LANE_OPS_PER_TERM:.0f} FP32 lane-ops per term x {SM_MAX_MHZ_RECIPE:.0f} MHz"}
     if clocks.get("sm_mhz"):
         roofline["frac_at_sampled_clock"] = achieved / (peak * clocks["sm_mhz"] / SM_MAX_MHZ_RECIPE)
 

@@ -54,11 +54,14 @@ typedef enum {
 } kvdro_status;
 
 typedef enum {
-    KVDRO_FP32 = 0,      /* per-term arithmetic in FP32; sums folded into FP64 */
+    KVDRO_FP32 = 0,      /* FP32 outputs.  When every L_max <= 2^22 they are the KVDRO_EXACT
+                            results rounded to FP32 (the exact kernel is also the fastest);
+                            otherwise per-term arithmetic in FP32 with sums folded into FP64 */
     KVDRO_FP64 = 1,      /* per-term arithmetic and sums in FP64 */
-    KVDRO_EXACT = 2,     /* per-term FP32 decisions on exact integer thresholds, exact integer
-                            counts and sample sums, combined once per cell in FP64; results
-                            carry FP64 rounding only.  Needs every L_max <= 2^22. */
+    KVDRO_EXACT = 2,     /* per term, FP32 integer arithmetic on exact integer thresholds
+                            (|x + 1 - t| summed exactly); exact integer counts and sums combined
+                            once per cell in FP64, so results carry FP64 rounding only.  Needs
+                            every L_max <= 2^22. */
     KVDRO_ENVELOPE = 3   /* not per term: each cell's sample sum from the sorted samples'
                             cumulative counts and sums at its exact threshold, O(1) per cell,
                             FP64 outputs with FP64 rounding only */
@@ -96,7 +99,7 @@ int kvdro_quantiles(kvdro_ctx* ctx, int32_t F, const double* fractiles, int32_t*
  * KVDRO_FP32 and double for the other modes.
  *   R, r       host int32[R], 1 <= R <= 2^20; every r must satisfy L_in_k <= r <= L_in_k + L_k for
  *              every class (the reservation domain of Sec. 2.2).
- *   NL, lam    host double[NL], finite, >= 0; 1 <= NL <= 256 (FP32, ENVELOPE) or 128 (FP64, EXACT).
+ *   NL, lam    host double[NL], finite, >= 0; 1 <= NL <= 256 (128 for KVDRO_FP64).
  *   E, eps     host double[E], finite, >= 0; 1 <= E <= 64.
  *   M, c_p,c_w host double[M] each, finite, >= 0; 1 <= M <= 65536.
  * Outputs (each may be NULL to skip it; host or device):

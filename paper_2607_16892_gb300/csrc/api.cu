@@ -426,11 +426,14 @@ int kvdro_eval_grid(kvdro_ctx* ctx, int precision, int32_t R, const int32_t* r, 
     const Prec P = precision == KVDRO_FP32 ? Prec::F32
                  : precision == KVDRO_FP64 ? Prec::F64
                  : precision == KVDRO_EXACT ? Prec::EXACT : Prec::ENVELOPE;
-    const int32_t maxNL = (P == Prec::F32 || P == Prec::ENVELOPE) ? kMaxNLf32 : kMaxNLf64;
-    if (P == Prec::EXACT)
-        for (int32_t k = 0; k < ctx->K; k++)
-            if (ctx->L[k] > kvdro::kExactMaxL)
-                return fail(ctx, KVDRO_EINVAL, "KVDRO_EXACT needs L_max <= 2^22 (class %d has %d)", k, ctx->L[k]);
+    const int32_t maxNL = P == Prec::F64 ? kMaxNLf64 : kMaxNLf32;
+    bool exact_ok = true;  // every class's support fits the exact kernel's integer sums
+    for (int32_t k = 0; k < ctx->K; k++) exact_ok = exact_ok && ctx->L[k] <= kvdro::kExactMaxL;
+    if (P == Prec::EXACT && !exact_ok)
+        return fail(ctx, KVDRO_EINVAL, "KVDRO_EXACT needs L_max <= 2^22 for every class");
+    // FP32 results come from the exact kernel (rounded to FP32) whenever it applies: it is exact
+    // and faster; the FP32-arithmetic kernel serves supports above 2^22.
+    const Prec KP = (P == Prec::F32 && exact_ok) ? Prec::EXACT : P;
     if (R < 1 || R > kMaxR) return fail(ctx, KVDRO_EINVAL, "R = %d outside [1, 2^20]", R);
     if (NL < 1 || NL > maxNL) return fail(ctx, KVDRO_EINVAL, "NL = %d outside [1, %d]", NL, maxNL);
     if (E < 1 || E > kMaxE) return fail(ctx, KVDRO_EINVAL, "E = %d outside [1, %d]", E, kMaxE);
@@ -452,7 +455,7 @@ int kvdro_eval_grid(kvdro_ctx* ctx, int precision, int32_t R, const int32_t* r, 
     ctx->last_stream = s;
 
     // Launch shape: lam tiles x r groups of warps per CTA.
-    const kvdro::GridShape shape = kvdro::grid_shape(P, R, NL, E);
+    const kvdro::GridShape shape = kvdro::grid_shape(KP, R, NL, E);
 
     // Grid parameters in one upload.
     const size_t gbytes = align_up((size_t)R * 4, 8) + 8 * ((size_t)NL + E + 2 * (size_t)M);
@@ -535,6 +538,7 @@ int kvdro_eval_grid(kvdro_ctx* ctx, int precision, int32_t R, const int32_t* r, 
     a.NL = NL;
     a.E = E;
     a.M = M;
+    a.f32_out = P == Prec::F32;
     a.S_out = outs[0].dev;
     a.cost_out = cost_dev;
     a.lam_idx_out = static_cast<int32_t*>(outs[2].dev);
@@ -547,7 +551,7 @@ int kvdro_eval_grid(kvdro_ctx* ctx, int precision, int32_t R, const int32_t* r, 
     for (int64_t m0 = 0; m0 < M; m0 += m_step) {
         a.m0 = (int32_t)m0;
         a.m_count = (int32_t)std::min<int64_t>(m_step, M - m0);
-        KV_CUDA(kvdro::launch_grid(P, shape, a, s), "grid kernel");
+        KV_CUDA(kvdro::launch_grid(KP, shape, a, s), "grid kernel");
     }
     KV_CUDA(cudaEventRecord(ctx->grid_t1, s), "recording grid end");
     ctx->grid_timed = true;

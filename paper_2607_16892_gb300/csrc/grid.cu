@@ -54,14 +54,16 @@ struct GridCfg {
     static_assert((V & (V - 1)) == 0 && V >= 2 && V <= 32, "tile must hold a power of two <= 32 cells");
     static_assert(P_ == Prec::F64 || TL_ % 2 == 0, "the FP32 and exact tiles pack lam values in pairs");
 };
-// FP32: 2 r x 8 lam tiles, up to 16 warps per CTA and two CTAs per SM (64 registers) for up to
-// 128 lam values; 2 x 16 tiles for 129..256 lam values.  FP64: 2 x 8 tiles.
-// All stage 4096-sample chunks (32 KB) through a 2-deep ring; the FP32 variants fold their
-// partial sums every 2 chunks (256 samples per lane) and unroll the sample loop 8 times.
+// 2 r x 8 lam tiles, up to 16 warps per CTA and (FP32, exact) two CTAs per SM (64 registers)
+// for up to 128 lam values; 2 x 16 tiles for 129..256 lam values.  FP64: 2 x 8 tiles.
+// All stage 4096-sample chunks (32 KB) through a 2-deep ring.  The FP32 variants fold their
+// partial sums every 2 chunks (256 samples per lane); the exact variants fold as often as their
+// support size requires.  The narrow variants unroll the sample loop 8 times.
 using CfgF32 = GridCfg<Prec::F32, 2, 8, 2, 2, 512, 4096, 2, 8>;
 using CfgF32Wide = GridCfg<Prec::F32, 2, 16, 2, 1, 512, 4096, 2, 2>;
 using CfgF64 = GridCfg<Prec::F64, 2, 8, 0, 1, 512, 4096, 2>;
-using CfgExact = GridCfg<Prec::EXACT, 2, 8, 0, 2, 512, 4096, 2>;
+using CfgExact = GridCfg<Prec::EXACT, 2, 8, 0, 2, 512, 4096, 2, 8>;
+using CfgExactWide = GridCfg<Prec::EXACT, 2, 16, 0, 1, 512, 4096, 2, 4>;
 constexpr int kWarpsTarget = 16;  // warps per CTA the r groups fill up to
 
 // ---------------------------------------------------------------- PTX helpers
@@ -90,24 +92,14 @@ __device__ __forceinline__ float relu(float w) {
     asm("max.f32 %0, %1, 0f00000000;" : "=f"(d) : "f"(w));
     return d;
 }
+__device__ __forceinline__ u64 abs2(u64 v) {
+    float a, b;
+    upk(v, a, b);
+    return pk(fabsf(a), fabsf(b));
+}
 __device__ __forceinline__ double relu(double w) {
     double d;
     asm("max.f64 %0, %1, 0d0000000000000000;" : "=d"(d) : "d"(w));
-    return d;
-}
-
-// min(max(a + b, 0), 1) in one FMA-pipe instruction.  With a an integer sample and b = 1 - t for
-// an integer threshold t this is exactly the indicator [a >= t]: a + 1 - t is an integer, >= 1
-// when a >= t and <= 0 otherwise, and rounding cannot move an integer across that gap.
-__device__ __forceinline__ float sat_add(float a, float b) {
-    float d;
-    asm("add.rn.sat.f32 %0, %1, %2;" : "=f"(d) : "f"(a), "f"(b));
-    return d;
-}
-// max(x, -2): padding samples (NaN) become -2, below every threshold; real samples (>= 0) pass.
-__device__ __forceinline__ float clamp_pad(float x) {
-    float d;
-    asm("max.f32 %0, %1, 0fC0000000;" : "=f"(d) : "f"(x));
     return d;
 }
 
@@ -431,10 +423,14 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
             acc64 = transpose_reduce<double, V>(vals, lane);
         }
     } else {
-        // EXACT: per cell (i, j), the active samples are those with x >= t_ij; the kernel counts them
-        // and sums them exactly (FP32 holds every integer below 2^24), and the epilogue forms
+        // EXACT: per cell (i, j) the active samples are x >= t_ij for an integer threshold t_ij, and
+        // sum_n max(kappa x_n + d, 0) = kappa sum_{x >= t} x + d #{x >= t}.  With y = x + 1 - t (an
+        // integer, exact in FP32) max(y, 0) = (y + |y|) / 2, and sum_n y has a closed form, so each
+        // term costs two packed adds: y, then the running sum of |y| (the absolute value rides on
+        // the add's operand).  Sums stay integers below 2^24 between folds into int64, hence exact.
+        // The count #{x >= t} comes from the class's cumulative counts; the epilogue forms
         // kappa * sum + d * count in FP64.
-        u64 nt[TR][TL / 2], sx[TR][TL / 2], cn[TR][TL / 2];  // nt holds 1 - t per cell
+        u64 nt[TR][TL / 2], acc[TR][TL / 2];  // nt holds 1 - t per cell
 #pragma unroll
         for (int jp = 0; jp < TL / 2; jp++) {
             const int j0 = lt * TL + 2 * jp;
@@ -444,36 +440,33 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
             const double k0 = mu0 + fmin(l0, cw), k1 = mu1 + fmin(l1, cw);
 #pragma unroll
             for (int i = 0; i < TR; i++) {
-                const float t0 = (v0 && rvalid[i]) ? exact_threshold(k0, (cp - mu0) * Lk - (cp + cw) * eta[i]) : 8388608.0f;
-                const float t1 = (v1 && rvalid[i]) ? exact_threshold(k1, (cp - mu1) * Lk - (cp + cw) * eta[i]) : 8388608.0f;
+                float t0 = (v0 && rvalid[i]) ? exact_threshold(k0, (cp - mu0) * Lk - (cp + cw) * eta[i]) : 8388608.0f;
+                float t1 = (v1 && rvalid[i]) ? exact_threshold(k1, (cp - mu1) * Lk - (cp + cw) * eta[i]) : 8388608.0f;
+                t0 = fminf(t0, (float)(a.L[k] + 1));  // no sample exceeds L: t = L + 1 means "none"
+                t1 = fminf(t1, (float)(a.L[k] + 1));
                 nt[i][jp] = pk(1.0f - t0, 1.0f - t1);
-                sx[i][jp] = 0ull;
-                cn[i][jp] = 0ull;
+                acc[i][jp] = 0ull;
             }
         }
-        // Fold the FP32 sums into int64 after `fe` loads of two samples: per-lane sums stay below
-        // 2 * fe * L <= 2^23 (fe is a power of two, the same for every thread of the CTA).
+        // Fold the FP32 sums into int64 after `fe` loads of two samples.  Every term is an integer
+        // in [0, L + 2], so a lane's sums stay below 2 fe (L + 2) <= 2^24 and are exact; fe is a
+        // power of two, the same for every thread of the CTA.
         int fe = 1;
-        while (fe < 1024 && 2 * (int64_t)(2 * fe) * a.L[k] <= (1ll << 23)) fe <<= 1;
-        long long acc_sx = 0, acc_cn = 0;
+        while (fe < 1024 && 2 * (int64_t)(2 * fe) * (a.L[k] + 2) <= (1ll << 24)) fe <<= 1;
+        long long acc_r = 0;
         auto fold = [&]() {
-            int vs[V], vc[V];
+            int vs[V];
 #pragma unroll
             for (int i = 0; i < TR; i++)
 #pragma unroll
                 for (int jp = 0; jp < TL / 2; jp++) {
-                    float a0, a1, b0, b1;
-                    upk(sx[i][jp], a0, a1);
-                    upk(cn[i][jp], b0, b1);
+                    float a0, a1;
+                    upk(acc[i][jp], a0, a1);
                     vs[i * TL + 2 * jp] = __float2int_rn(a0);
                     vs[i * TL + 2 * jp + 1] = __float2int_rn(a1);
-                    vc[i * TL + 2 * jp] = __float2int_rn(b0);
-                    vc[i * TL + 2 * jp + 1] = __float2int_rn(b1);
-                    sx[i][jp] = 0ull;
-                    cn[i][jp] = 0ull;
+                    acc[i][jp] = 0ull;
                 }
-            acc_sx += (long long)transpose_reduce<int, V>(vs, lane);
-            acc_cn += (long long)transpose_reduce<int, V>(vc, lane);
+            acc_r += (long long)transpose_reduce<int, V>(vs, lane);
         };
         int pending = 0;  // loads since the last fold
         for (int c = 0; c < nchunks; c++) {
@@ -485,21 +478,16 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
                 const int nq = cnt >> 6;
                 for (int t0 = 0; t0 < nq; t0 += fe) {
                     const int t1 = min(nq, t0 + fe);
+#pragma unroll(C::UNROLL)
                     for (int t = t0; t < t1; t++) {
                         const float4 v = q[lane + 32 * t];
-                        const float xa0 = clamp_pad(v.x), xa1 = clamp_pad(v.y);
-                        const float xb0 = clamp_pad(v.z), xb1 = clamp_pad(v.w);
-                        const u64 xa = pk(xa0, xa1), xb = pk(xb0, xb1);
+                        const float x0 = relu(v.x), x1 = relu(v.z);  // padding samples (NaN) become 0
+                        const u64 xa = pk(x0, x0), xb = pk(x1, x1);
 #pragma unroll
                         for (int i = 0; i < TR; i++)
 #pragma unroll
                             for (int jp = 0; jp < TL / 2; jp++) {
-                                float n0, n1;
-                                upk(nt[i][jp], n0, n1);
-                                const u64 pa = pk(sat_add(xa0, n0), sat_add(xa1, n1));
-                                const u64 pb = pk(sat_add(xb0, n0), sat_add(xb1, n1));
-                                sx[i][jp] = ffma2(pb, xb, ffma2(pa, xa, sx[i][jp]));
-                                cn[i][jp] = fadd2(cn[i][jp], fadd2(pa, pb));
+                                acc[i][jp] = fadd2(acc[i][jp], fadd2(abs2(fadd2(xa, nt[i][jp])), abs2(fadd2(xb, nt[i][jp]))));
                             }
                     }
                     pending += t1 - t0;
@@ -524,14 +512,34 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
         }
         if (!timeout) {
             if (pending > 0) fold();
-            // this lane's cell: kappa * sum + d * count in FP64
+            // this lane's cell: its threshold, the active count from the cumulative counts, then
+            // kappa * sum + d * count in FP64
             const int cidx = lane >> (5 - LOG2V);
             const int i = cidx / TL, j = cidx % TL;
+            float n_sel = 0.0f;
+#pragma unroll
+            for (int ii = 0; ii < TR; ii++)
+#pragma unroll
+                for (int jp = 0; jp < TL / 2; jp++) {
+                    float n0, n1;
+                    upk(nt[ii][jp], n0, n1);
+                    if (cidx == ii * TL + 2 * jp) n_sel = n0;
+                    if (cidx == ii * TL + 2 * jp + 1) n_sel = n1;
+                }
+            const long long t = 1 - (long long)n_sel;  // integer in [-1, 2^23]
+            const long long Nk = a.N[k];
+            const long long count = t <= 0 ? Nk : (t > a.L[k] ? 0 : Nk - (long long)a.cdf[a.hist_off[k] + t - 1]);
+            // acc_r = sum |x + 1 - t| over the samples and the padding zeros; relu = (y + |y|) / 2
+            const long long npad = np - Nk;
+            const long long sum_abs = acc_r - npad * (t > 1 ? t - 1 : 1 - t);
+            const long long sum_y = a.sumx[k] + Nk * (1 - t);
+            const long long sum_relu = (sum_y + sum_abs) / 2;  // each sample adds y + |y| = 2 relu(y)
+            const long long sum = sum_relu + (t - 1) * count;
             const int lj = lt * TL + j;
             const double l = lj < a.NL ? s_lam[lj] : 0.0;
             const double mu = fmin(l, cp), kap = mu + fmin(l, cw);
             const double d = (cp - mu) * Lk - (cp + cw) * eta[i];
-            acc64 = kap * (double)acc_sx + d * (double)acc_cn;
+            acc64 = kap * (double)sum + d * (double)count;
         }
     }
 
@@ -561,14 +569,15 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
             s_S[(r_local0 + i) * NLpad + lj] = S;
             if (a.S_out) {
                 const size_t o = (((size_t)m * a.K + k) * a.R + ri) * a.NL + lj;
-                if constexpr (P == Prec::F32) static_cast<float*>(a.S_out)[o] = (float)S;
-                else static_cast<double*>(a.S_out)[o] = S;  // F64 and EXACT
+                if (P == Prec::F32 || a.f32_out) static_cast<float*>(a.S_out)[o] = (float)S;
+                else static_cast<double*>(a.S_out)[o] = S;
             }
         }
     }
     __syncthreads();
 
-    cta_epilogue<P == Prec::F32>(a, s_S, s_lam, s_eps, NLpad, a.RG * TR, r_cta0, m, k);
+    if (P == Prec::F32 || a.f32_out) cta_epilogue<true>(a, s_S, s_lam, s_eps, NLpad, a.RG * TR, r_cta0, m, k);
+    else cta_epilogue<false>(a, s_S, s_lam, s_eps, NLpad, a.RG * TR, r_cta0, m, k);
 }
 
 // The same cells in O(1) each from the class's cumulative counts C[v] = #{x <= v} and sums
@@ -673,7 +682,8 @@ GridShape grid_shape(Prec p, int32_t R, int32_t NL, int32_t E) {
         return sh;
     }
     if (p == Prec::F64) return shape_for<CfgF64>(2, R, NL, E);
-    if (p == Prec::EXACT) return shape_for<CfgExact>(3, R, NL, E);
+    if (p == Prec::EXACT)
+        return NL <= kWarpsTarget * CfgExact::TL ? shape_for<CfgExact>(3, R, NL, E) : shape_for<CfgExactWide>(5, R, NL, E);
     if (NL <= kWarpsTarget * CfgF32::TL) return shape_for<CfgF32>(0, R, NL, E);
     return shape_for<CfgF32Wide>(1, R, NL, E);
 }
@@ -682,7 +692,11 @@ cudaError_t grid_prepare(Prec p) {
     // the largest layout any variant can need: 16 warps, 256 lam, 64 eps
     const int mx = (int)(smem_layout(16, 2, 256, 64, 4096, 4).total + 4096);
     if (p == Prec::F64) return cudaFuncSetAttribute(k_grid<CfgF64>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
-    if (p == Prec::EXACT) return cudaFuncSetAttribute(k_grid<CfgExact>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
+    if (p == Prec::EXACT) {
+        cudaError_t e = cudaFuncSetAttribute(k_grid<CfgExact>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
+        if (e != cudaSuccess) return e;
+        return cudaFuncSetAttribute(k_grid<CfgExactWide>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
+    }
     if (p == Prec::ENVELOPE)
         return cudaFuncSetAttribute(k_envelope, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                     (int)(8 * (256 + 64 + (size_t)kEnvR * 256)));
@@ -699,7 +713,8 @@ cudaError_t launch_grid(Prec p, const GridShape& sh, GridArgs a, cudaStream_t s)
     if (nblocks <= 0 || nblocks > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
     if (p == Prec::ENVELOPE) k_envelope<<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
     else if (p == Prec::F64) k_grid<CfgF64><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
-    else if (p == Prec::EXACT) k_grid<CfgExact><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
+    else if (p == Prec::EXACT && sh.variant == 3) k_grid<CfgExact><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
+    else if (p == Prec::EXACT) k_grid<CfgExactWide><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
     else if (sh.variant == 0) k_grid<CfgF32><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
     else k_grid<CfgF32Wide><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
     return cudaGetLastError();

@@ -43,7 +43,7 @@ cudaError_t launch_gather_quantiles(const int32_t* sorted, const int64_t* offset
 // threshold decisions with exact integer count and sample-sum accumulation, combined in FP64.
 // ENVELOPE: the same sums in O(1) per cell from cumulative counts and sums (not per term).
 enum class Prec { F32 = 0, F64 = 1, EXACT = 2, ENVELOPE = 3 };
-constexpr int32_t kExactMaxL = 1 << 22;  // EXACT needs 2 * L < 2^23 per fold of two samples
+constexpr int32_t kExactMaxL = 1 << 22;  // the exact kernel's integer sums need L <= 2^22
 
 struct GridArgs {
     const float2* pairs;        // padded (x, x) pairs
@@ -65,6 +65,7 @@ struct GridArgs {
     int32_t RG;                 // r groups per CTA
     int32_t r_blocks;           // CTAs per (m, k)
     int32_t m0, m_count;        // regime range covered by this launch
+    int32_t f32_out;            // exact kernel: write S, cost and the argmin keys as FP32 (FP32 mode)
     void* S_out;                // optional [M][K][R][NL]
     void* cost_out;             // [M][E][K][R] (caller's, or scratch for FP64 min_cost)
     int32_t* lam_idx_out;       // optional [M][E][K][R]

@@ -81,7 +81,7 @@ int setup_device(int dev, void** out, char* err, int32_t err_len) {
             cudaGetLastError();
             return report(err, err_len, KVDRO_ECUDA, "cudaGetSymbolAddress of the static scratch failed");
         }
-        if (kvdro::grid_prepare(kvdro::Prec::F32) != cudaSuccess) {
+        if (kvdro::grid_prepare(kvdro::Prec::F32) != cudaSuccess || kvdro::grid_prepare(kvdro::Prec::EXACT) != cudaSuccess) {
             cudaGetLastError();
             return report(err, err_len, KVDRO_ECUDA, "setting the grid kernel's shared-memory limit failed");
         }
@@ -252,8 +252,12 @@ extern "C" int kvdro_eval_grid_noalloc(int32_t K, const int64_t* offsets, const 
     NA_CUDA(cudaStreamSynchronize(s));
     if (bad) return report(err, err_len, KVDRO_EINVAL, "samples outside [0, L_max] of their class");
 
-    // ---- the FP32 grid kernel and the argmin finalisation
-    const kvdro::GridShape shape = kvdro::grid_shape(kvdro::Prec::F32, R, NL, E);
+    // ---- the grid kernel (the exact one, FP32 outputs, whenever every support is at most 2^22;
+    // else the FP32-arithmetic one) and the argmin finalisation
+    bool exact_ok = true;
+    for (int32_t k = 0; k < K; k++) exact_ok = exact_ok && L_max[k] <= kvdro::kExactMaxL;
+    const kvdro::Prec kp = exact_ok ? kvdro::Prec::EXACT : kvdro::Prec::F32;
+    const kvdro::GridShape shape = kvdro::grid_shape(kp, R, NL, E);
     kvdro::GridArgs a;
     a.pairs = sa.pairs;
     a.pair_off = sa.pair_off;
@@ -274,6 +278,7 @@ extern "C" int kvdro_eval_grid_noalloc(int32_t K, const int64_t* offsets, const 
     a.NL = NL;
     a.E = E;
     a.M = M;
+    a.f32_out = 1;
     a.S_out = nullptr;
     a.cost_out = cost;
     a.lam_idx_out = lam_idx;
@@ -284,7 +289,7 @@ extern "C" int kvdro_eval_grid_noalloc(int32_t K, const int64_t* offsets, const 
     for (int64_t m0 = 0; m0 < M; m0 += m_step) {
         a.m0 = (int32_t)m0;
         a.m_count = (int32_t)(m_step < M - m0 ? m_step : M - m0);
-        NA_CUDA(kvdro::launch_grid(kvdro::Prec::F32, shape, a, s));
+        NA_CUDA(kvdro::launch_grid(kp, shape, a, s));
     }
     kvdro::FinalizeArgs fa;
     fa.keys = a.keys;

@@ -68,7 +68,7 @@ def test_lognormal_k3_n1e3_full_grid(prec):
 
 @pytest.mark.parametrize("prec", ["fp64", "fp32", "exact"])
 def test_max_lambda_grid_and_single_points(prec):
-    nl = 256 if prec == "fp32" else 128
+    nl = 128 if prec == "fp64" else 256
     rng = np.random.default_rng(5)
     w = make([rng.integers(0, 500, 3000), rng.integers(200, 501, 17)], 500, [0, 250, 500],
              np.logspace(-4, 3, nl), [0.0, 40.0], [15.0, 2.0], [1.0, 0.5])
@@ -220,5 +220,16 @@ def test_exact_mode_rejects_support_above_its_limit():
         ev = lambda p: kvdro.kvdro_eval_grid(ctx, p, 1, [3], 1, [1.0], 1, [0.0], 1, [2.0], [1.0])
         assert _status(ev, kvdro.KVDRO_EXACT) == kvdro.KVDRO_EINVAL
         ev(kvdro.KVDRO_FP64)  # the other modes accept it
+        ev(kvdro.KVDRO_FP32)
     finally:
         kvdro.kvdro_destroy(ctx)
+
+
+@pytest.mark.parametrize("nl", [40, 200])
+def test_fp32_above_the_exact_limit_matches_the_oracle(nl):
+    """Supports above 2^22 take the FP32-arithmetic kernel (the exact one needs L <= 2^22)."""
+    L = (1 << 22) + 4096
+    rng = np.random.default_rng(11)
+    w = make([rng.integers(0, L + 1, 3000), np.concatenate([[0, L], rng.integers(L - 5000, L + 1, 300)])], L,
+             [1, 1 << 21, L - 2, L], np.logspace(-3, 2, nl), [0.0, 1000.0], [10.0, 1.0], [1.0, 1.0])
+    compare_full(w, run(w, kvdro.KVDRO_FP32), O.solve(w), "fp32")
