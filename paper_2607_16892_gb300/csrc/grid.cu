@@ -431,23 +431,27 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
         // The count #{x >= t} comes from the class's cumulative counts; the epilogue forms
         // kappa * sum + d * count in FP64.
         u64 nt[TR][TL / 2], acc[TR][TL / 2];  // nt holds 1 - t per cell
+        // Each lane works out the threshold of the cell it owns after the final transposition
+        // (cell lane >> (5 - LOG2V)); the warp's V thresholds then reach every lane by shuffles.
+        const int cidx = lane >> (5 - LOG2V);
+        const int ci = cidx / TL, cj = cidx % TL;
+        const int c_ri = r_cta0 + r_local0 + ci, c_lj = lt * TL + cj;
+        const bool c_valid = c_ri < a.R && c_lj < a.NL;
+        const double c_lam = s_lam[c_lj];  // s_lam is padded with zeros to NLpad
+        const double c_mu = fmin(c_lam, cp), c_kap = c_mu + fmin(c_lam, cw);
+        const double c_eta = c_valid ? (double)a.r[c_ri] - (double)a.L_in[k] : 0.0;
+        const double c_d = (cp - c_mu) * Lk - (cp + cw) * c_eta;
+        // no sample exceeds L, so t = L + 1 means "none" (and keeps |x + 1 - t| <= L + 2)
+        const float c_t = fminf(c_valid ? exact_threshold(c_kap, c_d) : 8388608.0f, (float)(a.L[k] + 1));
 #pragma unroll
-        for (int jp = 0; jp < TL / 2; jp++) {
-            const int j0 = lt * TL + 2 * jp;
-            const double l0 = s_lam[j0], l1 = s_lam[j0 + 1];
-            const bool v0 = j0 < a.NL, v1 = j0 + 1 < a.NL;
-            const double mu0 = fmin(l0, cp), mu1 = fmin(l1, cp);
-            const double k0 = mu0 + fmin(l0, cw), k1 = mu1 + fmin(l1, cw);
+        for (int i = 0; i < TR; i++)
 #pragma unroll
-            for (int i = 0; i < TR; i++) {
-                float t0 = (v0 && rvalid[i]) ? exact_threshold(k0, (cp - mu0) * Lk - (cp + cw) * eta[i]) : 8388608.0f;
-                float t1 = (v1 && rvalid[i]) ? exact_threshold(k1, (cp - mu1) * Lk - (cp + cw) * eta[i]) : 8388608.0f;
-                t0 = fminf(t0, (float)(a.L[k] + 1));  // no sample exceeds L: t = L + 1 means "none"
-                t1 = fminf(t1, (float)(a.L[k] + 1));
+            for (int jp = 0; jp < TL / 2; jp++) {
+                const float t0 = __shfl_sync(0xffffffffu, c_t, (i * TL + 2 * jp) << (5 - LOG2V));
+                const float t1 = __shfl_sync(0xffffffffu, c_t, (i * TL + 2 * jp + 1) << (5 - LOG2V));
                 nt[i][jp] = pk(1.0f - t0, 1.0f - t1);
                 acc[i][jp] = 0ull;
             }
-        }
         // Fold the FP32 sums into int64 after `fe` loads of two samples.  Every term is an integer
         // in [0, L + 2], so a lane's sums stay below 2 fe (L + 2) <= 2^24 and are exact; fe is a
         // power of two, the same for every thread of the CTA.
@@ -512,21 +516,9 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
         }
         if (!timeout) {
             if (pending > 0) fold();
-            // this lane's cell: its threshold, the active count from the cumulative counts, then
+            // this lane's cell: the active count from the cumulative counts, then
             // kappa * sum + d * count in FP64
-            const int cidx = lane >> (5 - LOG2V);
-            const int i = cidx / TL, j = cidx % TL;
-            float n_sel = 0.0f;
-#pragma unroll
-            for (int ii = 0; ii < TR; ii++)
-#pragma unroll
-                for (int jp = 0; jp < TL / 2; jp++) {
-                    float n0, n1;
-                    upk(nt[ii][jp], n0, n1);
-                    if (cidx == ii * TL + 2 * jp) n_sel = n0;
-                    if (cidx == ii * TL + 2 * jp + 1) n_sel = n1;
-                }
-            const long long t = 1 - (long long)n_sel;  // integer in [-1, 2^23]
+            const long long t = (long long)c_t;  // integer in [-1, L + 1]
             const long long Nk = a.N[k];
             const long long count = t <= 0 ? Nk : (t > a.L[k] ? 0 : Nk - (long long)a.cdf[a.hist_off[k] + t - 1]);
             // acc_r = sum |x + 1 - t| over the samples and the padding zeros; relu = (y + |y|) / 2
@@ -535,10 +527,7 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
             const long long sum_y = a.sumx[k] + Nk * (1 - t);
             const long long sum_relu = (sum_y + sum_abs) / 2;  // each sample adds y + |y| = 2 relu(y)
             const long long sum = sum_relu + (t - 1) * count;
-            const int lj = lt * TL + j;
-            const double l = lj < a.NL ? s_lam[lj] : 0.0;
-            const double mu = fmin(l, cp), kap = mu + fmin(l, cw);
-            const double d = (cp - mu) * Lk - (cp + cw) * eta[i];
+            const double kap = c_kap, d = c_d;
             acc64 = kap * (double)sum + d * (double)count;
         }
     }
