@@ -36,28 +36,20 @@ __device__ __forceinline__ void tail(const ClassView& c, int64_t t, int64_t& cnt
     sum = c.sumx - below_s;
 }
 
-__device__ __forceinline__ int64_t threshold(double kap, double d, int32_t L) {
-    if (kap > 0.0) {
-        const double xs = floor(-d / kap) + 1.0;
-        return xs <= 0.0 ? 0 : (xs >= (double)L + 1.0 ? (int64_t)L + 1 : (int64_t)xs);
-    }
-    return d > 0.0 ? 0 : (int64_t)L + 1;
-}
-
 // g(gamma) and its right derivative.
 __device__ __forceinline__ void g_and_slope(const ClassView& c, double eta, double cp, double cw, double eps, double gam,
-                                            double& g, double& slope) {
+                                            double inv_n, double& g, double& slope) {
     const double mu = fmin(gam, cp), nu = fmin(gam, cw), kap = mu + nu;
     const double dmu = gam < cp ? 1.0 : 0.0, dnu = gam < cw ? 1.0 : 0.0;
     const double L = (double)c.L, N = (double)c.N;
     const double d = (cp - mu) * L - (cp + cw) * eta;
     int64_t cnt, sum;
-    tail(c, threshold(kap, d, c.L), cnt, sum);
+    tail(c, first_active(kap, d, c.L), cnt, sum);
     const double tot = N * cw * eta - nu * (double)c.sumx + kap * (double)sum + d * (double)cnt;
-    g = gam * eps + tot / N;
+    g = gam * eps + tot * inv_n;
     // right derivative: the active set just above gamma is the one at gamma up to samples whose
     // excess is exactly zero, which change the value by nothing and the slope only at a kink
-    slope = eps + (-dnu * (double)c.sumx + (dmu + dnu) * (double)sum - dmu * L * (double)cnt) / N;
+    slope = eps + (-dnu * (double)c.sumx + (dmu + dnu) * (double)sum - dmu * L * (double)cnt) * inv_n;
 }
 
 __global__ void __launch_bounds__(kDualThreads) k_dual(const DualArgs a) {
@@ -79,16 +71,17 @@ __global__ void __launch_bounds__(kDualThreads) k_dual(const DualArgs a) {
     c.L = a.L[k];
     const double cp = a.cp[m], cw = a.cw[m], eps = a.eps[e];
     const double eta = (double)a.r[ri] - (double)a.L_in[k];
+    const double inv_n = 1.0 / (double)c.N;
     double lo = 0.0, hi = fmax(cp, cw), g_lo, s_lo, g_hi, s_hi;
-    g_and_slope(c, eta, cp, cw, eps, lo, g_lo, s_lo);
+    g_and_slope(c, eta, cp, cw, eps, lo, inv_n, g_lo, s_lo);
     double best_g = g_lo, best_gam = lo;
     if (s_lo < 0.0 && hi > 0.0) {
-        g_and_slope(c, eta, cp, cw, eps, hi, g_hi, s_hi);
+        g_and_slope(c, eta, cp, cw, eps, hi, inv_n, g_hi, s_hi);
         for (int it = 0; it < kBisections; it++) {
             const double mid = 0.5 * (lo + hi);
             if (!(mid > lo && mid < hi)) break;
             double gm, sm;
-            g_and_slope(c, eta, cp, cw, eps, mid, gm, sm);
+            g_and_slope(c, eta, cp, cw, eps, mid, inv_n, gm, sm);
             if (sm >= 0.0) { hi = mid; g_hi = gm; }
             else { lo = mid; g_lo = gm; }
         }

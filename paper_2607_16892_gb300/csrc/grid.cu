@@ -103,17 +103,6 @@ __device__ __forceinline__ double relu(double w) {
     return d;
 }
 
-// Smallest integer t with kappa * t + d > 0, clamped to [-1, 2^23] (so 1 - t is exact in FP32).
-// For integer samples x <= 2^22, x >= t exactly when max(kappa x + d, 0) is positive; a sample
-// at the boundary has kappa x + d within a rounding of zero, so either choice adds nothing
-// material.  2^23 means "never active".
-__device__ __forceinline__ float exact_threshold(double kappa, double d) {
-    if (!(kappa > 0.0)) return d > 0.0 ? -1.0f : 8388608.0f;
-    double t = floor(-d / kappa) + 1.0;
-    t = fmin(fmax(t, -1.0), 8388608.0);
-    return (float)t;
-}
-
 __device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
 
 __device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
@@ -441,8 +430,8 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
         const double c_mu = fmin(c_lam, cp), c_kap = c_mu + fmin(c_lam, cw);
         const double c_eta = c_valid ? (double)a.r[c_ri] - (double)a.L_in[k] : 0.0;
         const double c_d = (cp - c_mu) * Lk - (cp + cw) * c_eta;
-        // no sample exceeds L, so t = L + 1 means "none" (and keeps |x + 1 - t| <= L + 2)
-        const float c_t = fminf(c_valid ? exact_threshold(c_kap, c_d) : 8388608.0f, (float)(a.L[k] + 1));
+        // t = L + 1 means "none" (no sample exceeds L); t in [0, L + 1] keeps |x + 1 - t| <= L + 1
+        const float c_t = (float)(c_valid ? first_active(c_kap, c_d, a.L[k]) : (int64_t)a.L[k] + 1);
 #pragma unroll
         for (int i = 0; i < TR; i++)
 #pragma unroll
@@ -518,7 +507,7 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
             if (pending > 0) fold();
             // this lane's cell: the active count from the cumulative counts, then
             // kappa * sum + d * count in FP64
-            const long long t = (long long)c_t;  // integer in [-1, L + 1]
+            const long long t = (long long)c_t;  // integer in [0, L + 1]
             const long long Nk = a.N[k];
             const long long count = t <= 0 ? Nk : (t > a.L[k] ? 0 : Nk - (long long)a.cdf[a.hist_off[k] + t - 1]);
             // acc_r = sum |x + 1 - t| over the samples and the padding zeros; relu = (y + |y|) / 2
@@ -592,7 +581,7 @@ __global__ void __launch_bounds__(kEnvThreads) k_envelope(const GridArgs a) {
     const double cp = a.cp[m], cw = a.cw[m];
     const int32_t Lk = a.L[k];
     const int64_t Nk = a.N[k];
-    const double N = (double)Nk, sumx = (double)a.sumx[k];
+    const double N = (double)Nk, sumx = (double)a.sumx[k], inv_n = 1.0 / N;
     const int32_t* C = a.cdf + a.hist_off[k];
     const int64_t* CS = a.csum + a.hist_off[k];
     for (int cell = threadIdx.x; cell < kEnvR * a.NL; cell += blockDim.x) {
@@ -603,17 +592,11 @@ __global__ void __launch_bounds__(kEnvThreads) k_envelope(const GridArgs a) {
         const double lam = s_lam[j];
         const double mu = fmin(lam, cp), nu = fmin(lam, cw), kap = mu + nu;
         const double d = (cp - mu) * (double)Lk - (cp + cw) * eta;
-        int64_t t;  // first active sample value, clamped to [0, L + 1]
-        if (kap > 0.0) {
-            const double xs = floor(-d / kap) + 1.0;
-            t = xs <= 0.0 ? 0 : (xs >= (double)Lk + 1.0 ? (int64_t)Lk + 1 : (int64_t)xs);
-        } else {
-            t = d > 0.0 ? 0 : (int64_t)Lk + 1;
-        }
+        const int64_t t = first_active(kap, d, Lk);  // first active sample value, in [0, L + 1]
         const int64_t below_n = t >= 1 ? (int64_t)C[t - 1] : 0;
         const int64_t below_s = t >= 1 ? CS[t - 1] : 0;
         const double tot = N * cw * eta - nu * sumx + kap * (double)(a.sumx[k] - below_s) + d * (double)(Nk - below_n);
-        const double S = tot / N;
+        const double S = tot * inv_n;
         s_S[rl * a.NL + j] = S;
         if (a.S_out) static_cast<double*>(a.S_out)[(((size_t)m * a.K + k) * a.R + ri) * a.NL + j] = S;
     }

@@ -123,4 +123,29 @@ struct DualArgs {
 };
 cudaError_t launch_dual(const DualArgs& a, cudaStream_t s);
 
+
+#ifdef __CUDACC__
+// The first active support point of a cell: the smallest integer t in [0, L] with
+// kappa * t + d > 0, or L + 1 when there is none (kappa >= 0, so the condition is monotone in
+// t).  One FMA gives the sign of kappa * t + d exactly, so each test is exact.  An FP32 estimate
+// of -d / kappa (off by a few units at most for L <= 2^24) is corrected by at most 8 such tests
+// each way; should that not settle it, the FP64 quotient is corrected the same way.
+__device__ __forceinline__ int64_t first_active(double kappa, double d, int64_t L) {
+    if (d > 0.0) return 0;
+    if (!(kappa > 0.0) || !(fma(kappa, (double)L, d) > 0.0)) return L + 1;
+    // here t is in [1, L]: kappa (t - 1) + d <= 0 < kappa t + d
+    auto settle = [&](double q, int64_t& t) {
+        const double e = floor(q) + 1.0;
+        t = e < 1.0 ? 1 : (e > (double)L ? L : (int64_t)e);
+        for (int i = 0; i < 8 && t > 1 && fma(kappa, (double)(t - 1), d) > 0.0; i++) t--;
+        for (int i = 0; i < 8 && t < L && !(fma(kappa, (double)t, d) > 0.0); i++) t++;
+        return (t == 1 || !(fma(kappa, (double)(t - 1), d) > 0.0)) && fma(kappa, (double)t, d) > 0.0;
+    };
+    int64_t t;
+    if (settle((double)__fdiv_rn(-(float)d, (float)kappa), t)) return t;
+    (void)settle(-d / kappa, t);
+    return t;
+}
+#endif
+
 }  // namespace kvdro
