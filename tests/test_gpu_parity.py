@@ -225,6 +225,18 @@ def test_exact_mode_rejects_support_above_its_limit():
         kvdro.kvdro_destroy(ctx)
 
 
+@pytest.mark.parametrize("prec", ["exact", "fp32"])
+def test_exact_kernel_at_its_largest_support(prec):
+    """L = 2^22, the largest support the exact kernel takes: its FP32 sums fold after every
+    load; samples at 0 and at L, cells with every sample active (lam = 0) and none active."""
+    L = 1 << 22
+    rng = np.random.default_rng(12)
+    w = make([np.concatenate([[0, 0, L, L], rng.integers(0, L + 1, 2500)]), rng.integers(L - 3000, L + 1, 700)], L,
+             [0, 1, 1 << 21, L - 1, L], np.concatenate([[0.0], np.logspace(-3, 2, 20)]), [0.0, 5000.0], [10.0, 0.5],
+             [1.0, 2.0])
+    compare_full(w, run(w, P[prec]), O.solve(w), prec)
+
+
 @pytest.mark.parametrize("nl", [40, 200])
 def test_fp32_above_the_exact_limit_matches_the_oracle(nl):
     """Supports above 2^22 take the FP32-arithmetic kernel (the exact one needs L <= 2^22)."""
