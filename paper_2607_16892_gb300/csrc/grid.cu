@@ -430,24 +430,22 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
         const double c_mu = fmin(c_lam, cp), c_kap = c_mu + fmin(c_lam, cw);
         const double c_eta = c_valid ? (double)a.r[c_ri] - (double)a.L_in[k] : 0.0;
         const double c_d = (cp - c_mu) * Lk - (cp + cw) * c_eta;
-        // t = L + 1 means "none" (no sample exceeds L).  The stream uses t_s = max(t, 1): samples
-        // equal to 0 add nothing to sum_{x >= t} x, and t_s in [1, L + 1] keeps |x + 1 - t_s| <= L.
-        const int64_t c_t = c_valid ? first_active(c_kap, c_d, a.L[k]) : (int64_t)a.L[k] + 1;
-        const float c_ts = (float)(c_t > 1 ? c_t : 1);
+        // t = L + 1 means "none" (no sample exceeds L); t in [0, L + 1] keeps |x + 1 - t| <= L + 1
+        const float c_t = (float)(c_valid ? first_active(c_kap, c_d, a.L[k]) : (int64_t)a.L[k] + 1);
 #pragma unroll
         for (int i = 0; i < TR; i++)
 #pragma unroll
             for (int jp = 0; jp < TL / 2; jp++) {
-                const float t0 = __shfl_sync(0xffffffffu, c_ts, (i * TL + 2 * jp) << (5 - LOG2V));
-                const float t1 = __shfl_sync(0xffffffffu, c_ts, (i * TL + 2 * jp + 1) << (5 - LOG2V));
+                const float t0 = __shfl_sync(0xffffffffu, c_t, (i * TL + 2 * jp) << (5 - LOG2V));
+                const float t1 = __shfl_sync(0xffffffffu, c_t, (i * TL + 2 * jp + 1) << (5 - LOG2V));
                 nt[i][jp] = pk(1.0f - t0, 1.0f - t1);
                 acc[i][jp] = 0ull;
             }
         // Fold the FP32 sums into int64 after `fe` loads of two samples.  Every term is an integer
-        // in [0, L], so a lane's sums stay at most 2 fe L <= 2^24 and are exact; fe is a power of
-        // two, the same for every thread of the CTA.
+        // in [0, L + 2], so a lane's sums stay below 2 fe (L + 2) <= 2^24 and are exact; fe is a
+        // power of two, the same for every thread of the CTA.
         int fe = 1;
-        while (fe < 1024 && 2 * (int64_t)(2 * fe) * a.L[k] <= (1ll << 24)) fe <<= 1;
+        while (fe < 1024 && 2 * (int64_t)(2 * fe) * (a.L[k] + 2) <= (1ll << 24)) fe <<= 1;
         long long acc_r = 0;
         auto fold = [&]() {
             int vs[V];
@@ -509,17 +507,15 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
             if (pending > 0) fold();
             // this lane's cell: the active count from the cumulative counts, then
             // kappa * sum + d * count in FP64
-            const long long t = c_t, ts = c_t > 1 ? c_t : 1;  // t in [0, L + 1], ts = max(t, 1)
+            const long long t = (long long)c_t;  // integer in [0, L + 1]
             const long long Nk = a.N[k];
-            const int32_t* C = a.cdf + a.hist_off[k];
-            const long long count = t <= 0 ? Nk : (t > a.L[k] ? 0 : Nk - (long long)C[t - 1]);
-            const long long count_s = ts > a.L[k] ? 0 : Nk - (long long)C[ts - 1];
-            // acc_r = sum |x + 1 - ts| over the samples and the padding zeros; relu = (y + |y|) / 2
+            const long long count = t <= 0 ? Nk : (t > a.L[k] ? 0 : Nk - (long long)a.cdf[a.hist_off[k] + t - 1]);
+            // acc_r = sum |x + 1 - t| over the samples and the padding zeros; relu = (y + |y|) / 2
             const long long npad = np - Nk;
-            const long long sum_abs = acc_r - npad * (ts - 1);
-            const long long sum_y = a.sumx[k] + Nk * (1 - ts);
+            const long long sum_abs = acc_r - npad * (t > 1 ? t - 1 : 1 - t);
+            const long long sum_y = a.sumx[k] + Nk * (1 - t);
             const long long sum_relu = (sum_y + sum_abs) / 2;  // each sample adds y + |y| = 2 relu(y)
-            const long long sum = sum_relu + (ts - 1) * count_s;  // sum_{x >= ts} x = sum_{x >= t} x
+            const long long sum = sum_relu + (t - 1) * count;
             const double kap = c_kap, d = c_d;
             acc64 = kap * (double)sum + d * (double)count;
         }
