@@ -33,6 +33,7 @@ constexpr int32_t kMaxE = 64;
 constexpr int32_t kMaxM = 65536;
 constexpr int32_t kMaxF = 65536;
 constexpr int64_t kMaxKF = 1 << 22;
+constexpr long long kTestWaitCycles = 2000000;  // the wait test's bound: about 1 ms at 2 GHz
 constexpr int32_t kMaxNLf32 = 256;
 constexpr int32_t kMaxNLf64 = 128;
 
@@ -47,6 +48,7 @@ struct kvdro_ctx {
     int device = 0;
     std::string err;
     int fail_after = -1;  // test hook: the fail_after-th allocation of this context fails
+    int skip_chunk = -1;  // test hook: grid kernels never copy this chunk, so their waits run out
     int allocs = 0;
     cudaStream_t last_stream = nullptr;
 
@@ -213,6 +215,7 @@ int kvdro_create(kvdro_ctx** out, int device_ordinal) {
     if (!ctx) return KVDRO_ENOMEM;
     ctx->device = device_ordinal;
     if (const char* f = std::getenv("KVDRO_TEST_FAIL_ALLOC")) ctx->fail_after = std::atoi(f);
+    if (const char* f = std::getenv("KVDRO_TEST_SKIP_CHUNK")) ctx->skip_chunk = std::atoi(f);
     DeviceGuard g(device_ordinal);
     if (!g.ok || kvdro::grid_prepare(Prec::F32) != cudaSuccess || kvdro::grid_prepare(Prec::F64) != cudaSuccess ||
         cudaEventCreateWithFlags(&ctx->pin_free, cudaEventDisableTiming) != cudaSuccess ||
@@ -547,6 +550,8 @@ int kvdro_eval_grid(kvdro_ctx* ctx, int precision, int32_t R, const int32_t* r, 
     const int64_t per_m = (int64_t)ctx->K * shape.r_blocks;
     const int64_t m_step = std::max<int64_t>(1, 0x7fffffffLL / per_m);
     ctx->grid_timed = false;
+    if (ctx->skip_chunk >= 0)  // test hook: bounded waits of about 1 ms that run out on one chunk
+        KV_CUDA(kvdro::set_wait_test(ctx->skip_chunk, kTestWaitCycles, s), "arming the wait test");
     KV_CUDA(cudaEventRecord(ctx->grid_t0, s), "recording grid start");
     for (int64_t m0 = 0; m0 < M; m0 += m_step) {
         a.m0 = (int32_t)m0;
@@ -554,6 +559,7 @@ int kvdro_eval_grid(kvdro_ctx* ctx, int precision, int32_t R, const int32_t* r, 
         KV_CUDA(kvdro::launch_grid(KP, shape, a, s), "grid kernel");
     }
     KV_CUDA(cudaEventRecord(ctx->grid_t1, s), "recording grid end");
+    if (ctx->skip_chunk >= 0) KV_CUDA(kvdro::set_wait_test(-1, 0, s), "disarming the wait test");
     ctx->grid_timed = true;
 
     kvdro::FinalizeArgs fa;

@@ -34,6 +34,10 @@ namespace {
 typedef unsigned long long u64;
 
 constexpr long long kWaitCycles = 4000000000LL;  // ~2 s at 2 GHz: bound on any barrier wait
+// The bound in force, and a test hook: a chunk index whose copy is never issued, so the waits
+// on its barrier run out (-1: none).  Set together by set_wait_test.
+__device__ long long g_wait_cycles = kWaitCycles;
+__device__ int g_test_skip_chunk = -1;
 
 constexpr int ilog2(int v) { return v <= 1 ? 0 : 1 + ilog2(v / 2); }
 
@@ -131,12 +135,12 @@ __device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
     return ok != 0;
 }
 
-// Wait for phase `parity` of `bar`; gives up after kWaitCycles and returns false.
+// Wait for phase `parity` of `bar`; gives up after g_wait_cycles and returns false.
 __device__ __noinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity) {
     if (mbar_try(bar, parity)) return true;
-    const long long t0 = clock64();
+    const long long t0 = clock64(), limit = g_wait_cycles;
     while (!mbar_try(bar, parity)) {
-        if (clock64() - t0 > kWaitCycles) return false;
+        if (clock64() - t0 > limit) return false;
     }
     return true;
 }
@@ -260,6 +264,7 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
     const int nchunks = (int)((np + C::CHUNK - 1) / C::CHUNK);
     const float2* src = a.pairs + pbase;
     auto issue = [&](int c) {
+        if (c == g_test_skip_chunk) return;  // test hook: nothing will complete this chunk's barrier
         const int s = c % C::STAGES;
         const int64_t cnt = min((int64_t)C::CHUNK, np - (int64_t)c * C::CHUNK);
         tma_bulk_load(smem_u32(ring + (size_t)s * C::CHUNK), src + (int64_t)c * C::CHUNK, (uint32_t)(cnt * sizeof(float2)),
@@ -675,6 +680,15 @@ cudaError_t grid_prepare(Prec p) {
     cudaError_t e = cudaFuncSetAttribute(k_grid<CfgF32>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
     if (e != cudaSuccess) return e;
     return cudaFuncSetAttribute(k_grid<CfgF32Wide>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
+}
+
+cudaError_t set_wait_test(int skip_chunk, long long wait_cycles, cudaStream_t s) {
+    const long long w = wait_cycles > 0 ? wait_cycles : kWaitCycles;
+    cudaError_t e = cudaMemcpyToSymbolAsync(g_test_skip_chunk, &skip_chunk, sizeof(int), 0, cudaMemcpyHostToDevice, s);
+    if (e != cudaSuccess) return e;
+    e = cudaMemcpyToSymbolAsync(g_wait_cycles, &w, sizeof(long long), 0, cudaMemcpyHostToDevice, s);
+    if (e != cudaSuccess) return e;
+    return cudaStreamSynchronize(s);  // the host values are on this stack frame
 }
 
 cudaError_t launch_grid(Prec p, const GridShape& sh, GridArgs a, cudaStream_t s) {

@@ -101,6 +101,9 @@ GridShape grid_shape(Prec p, int32_t R, int32_t NL, int32_t E);
 cudaError_t grid_prepare(Prec p);             // per-device attribute setup of every variant of p
 // Launches over regimes [a.m0, a.m0 + a.m_count); fills a.LT, a.RG, a.r_blocks from `sh`.
 cudaError_t launch_grid(Prec p, const GridShape& sh, GridArgs a, cudaStream_t s);
+// Test hook for the bounded waits of the grid kernel: skip_chunk >= 0 makes every CTA leave that
+// chunk's copy unissued, so its waits give up after wait_cycles; (-1, 0) restores the defaults.
+cudaError_t set_wait_test(int skip_chunk, long long wait_cycles, cudaStream_t s);
 cudaError_t launch_finalize(Prec p, const FinalizeArgs& a, cudaStream_t s);
 
 // dual.cu: exact minimisation over gamma >= 0 per (regime, radius, class, reservation)

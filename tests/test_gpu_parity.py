@@ -212,6 +212,36 @@ def test_injected_allocation_failure_reports_enomem(monkeypatch):
     kvdro.kvdro_destroy(ctx)
 
 
+@pytest.mark.parametrize("prec", ["fp32", "fp64"])
+def test_a_wait_that_runs_out_reports_etimeout_and_the_device_stays_usable(monkeypatch, prec):
+    """Failure detection without a fault: a test hook leaves one chunk's copy unissued, so nothing
+    completes that barrier; every CTA's bounded wait (about 1 ms under the hook) gives up, the CTA
+    drains the copies it did issue and sets the error bit, and the call reports KVDRO_ETIMEOUT.
+    Afterwards the same CUDA context evaluates correctly."""
+    rng = np.random.default_rng(3)
+    w = make([rng.integers(0, 900, 20000)], 1000, [10, 200, 600], [0.5, 5.0], [0.0, 10.0], 10.0, 1.0)  # 5 chunks
+    monkeypatch.setenv("KVDRO_TEST_SKIP_CHUNK", "2")
+    ctx = kvdro.kvdro_create(0)
+    monkeypatch.delenv("KVDRO_TEST_SKIP_CHUNK")
+    try:
+        kvdro.kvdro_load_samples(ctx, w.K, w.offsets, torch.from_numpy(w.samples).cuda(), w.L, w.L_in)
+        dt = np.float32 if prec == "fp32" else np.float64
+        cost = np.empty((1, 2, 1, 3), dt)  # host output: the call waits and reads the status
+        ev = lambda **kw: kvdro.kvdro_eval_grid(ctx, P[prec], 3, w.r, 2, w.lam, 2, w.eps, 1, w.cp, w.cw, **kw)
+        assert _status(ev, cost=cost) == kvdro.KVDRO_ETIMEOUT
+        assert "gave up waiting" in kvdro.kvdro_last_error(ctx)
+        r_idx = torch.empty((1, 2, 1), dtype=torch.int32, device="cuda")  # device output: kvdro_sync reports it
+        ev(r_idx=r_idx)
+        assert _status(kvdro.kvdro_sync, ctx) == kvdro.KVDRO_ETIMEOUT
+        assert _status(kvdro.kvdro_sync, ctx) == kvdro.KVDRO_OK  # reported once
+        # modes without staged copies are unaffected by the hook
+        kvdro.kvdro_eval_grid(ctx, kvdro.KVDRO_ENVELOPE, 3, w.r, 2, w.lam, 2, w.eps, 1, w.cp, w.cw, r_idx=r_idx)
+        kvdro.kvdro_sync(ctx)
+    finally:
+        kvdro.kvdro_destroy(ctx)
+    compare_full(w, run(w, P[prec]), O.solve(w), prec)  # a context without the hook, same device
+
+
 def test_exact_mode_rejects_support_above_its_limit():
     ctx = kvdro.kvdro_create(0)
     try:
