@@ -71,6 +71,8 @@ def parse_args():
                         "(--warmup untimed, --steps timed runs) and print one line per run")
     p.add_argument("--suite", action="store_true",
                    help="time every workload in each precision (one JSON line per case) instead of the contract line")
+    p.add_argument("--cpu-suite", action="store_true",
+                   help="time the CPU oracle (the reported baseline) on every workload, one line each")
     p.add_argument("--bcd", action="store_true",
                    help="time the block-coordinate descent (Alg. 1) on the scalability instances, one line each")
     return p.parse_args()
@@ -441,6 +443,56 @@ def run_suite(args):
                                                                 "terms_per_s")}}), flush=True)
 
 
+def run_cpu_suite(args):
+    """The CPU oracle -- the reported baseline, never tuned -- on every workload: the direct
+    per-term FP64 evaluation on all host cores and on one (the 3-class workload in full, 16 strided
+    (regime, class, r) rows of the others, every lam and sample), the envelope regrouping
+    (cells/s; a different algorithm), and its quantiles (a sort of every class)."""
+    from oracle import oracle as O
+    from synth import WORKLOADS
+
+    threads = O.default_threads()
+    for name in ("lognormal_k3_n1e3", "lognormal_k8_n1e5", "heavytail_k16_n1e6", "regimes_k8_n2e5", "drift_k32_n1e6"):
+        w = WORKLOADS[name]()
+        M, K, R, NL = len(w.cp), w.K, len(w.r), len(w.lam)
+        rows_all = M * K * R
+        full = name == "lognormal_k3_n1e3"
+        n_rows = rows_all if full else 16
+        pick = np.arange(rows_all) if full else np.linspace(0, rows_all - 1, n_rows).round().astype(np.int64)
+
+        def cells(rows):
+            m, rest = np.divmod(rows, K * R)
+            k, r = np.divmod(rest, R)
+            mm, ll = np.repeat(m, NL), np.tile(np.arange(NL), rows.size)
+            return mm.astype(np.int32), np.repeat(k, NL), np.repeat(r, NL), ll
+
+        def terms(rows):
+            _, rest = np.divmod(rows, K * R)
+            return int(sum(int(w.N[k]) for k in rest // R) * NL)
+
+        t0 = time.perf_counter()
+        O.eval_cells(w, *cells(pick), threads=threads)
+        t_all = time.perf_counter() - t0
+        one = pick[: max(1, min(pick.size, 2 if not full else pick.size))]
+        t0 = time.perf_counter()
+        O.eval_cells(w, *cells(one), threads=1)
+        t_one = time.perf_counter() - t0
+        we = w if M <= 16 else slice_workload(w, regimes=list(range(0, M, M // 16)), name=w.name)
+        t0 = time.perf_counter()
+        O.envelope_grid(we, threads=threads)
+        t_env = time.perf_counter() - t0
+        env_cells = len(we.cp) * K * R * NL
+        t0 = time.perf_counter()
+        O.quantiles(w, w.fractiles)
+        t_sort = time.perf_counter() - t0
+        print(json.dumps({"cpu_suite": True, "workload": w.name, "kind": "oracle",
+                          "direct_terms_per_s": terms(pick) / t_all, "direct_cores": threads,
+                          "direct_sample": f"{pick.size} (regime, class, r) rows x {NL} lam x all samples",
+                          "direct_terms_per_s_one_core": terms(one) / t_one,
+                          "envelope_cells_per_s": env_cells / t_env, "envelope_cells": env_cells,
+                          "sort_quantiles_s": t_sort, "samples": int(w.N.sum())}), flush=True)
+
+
 # BCD-DRO solve times of the paper's scalability table (Sec. 5.2; hardware unstated), by
 # (classes, configurations, samples per class): context for the host solve, not a target
 PAPER_BCD_SECONDS = {(3, 4, 100): 0.17, (4, 4, 150): 0.8, (5, 5, 200): 4.3, (6, 6, 300): 10.5, (8, 6, 500): 22.4,
@@ -507,6 +559,9 @@ def main():
     args = parse_args()
     if args.case:
         run_case(args)
+        return
+    if args.cpu_suite:
+        run_cpu_suite(args)
         return
     if args.bcd:
         run_bcd(args)
