@@ -50,7 +50,7 @@ LANE_OPS_PER_TERM = 2.0
 TERMS_PER_CLK_PER_SM = LANE_OPS_PER_CLK_PER_SM / LANE_OPS_PER_TERM
 GRID_SOURCE = os.path.join(ROOT, "paper_2607_16892_gb300", "csrc", "grid.cu")
 PROFILE = os.path.join(ROOT, "profiles", "k_grid_exact_lognormal_k8_n1e5.md")
-LAUNCHES_PER_STEP = 6  # histogram, scan, expand, quantile gather, grid, argmin finalise
+LAUNCHES_PER_STEP = 7  # histogram, scan totals, scan, expand, quantile gather, grid, argmin finalise
 # FP64 pipe bound of the native FP64 mode: per term one DFMA (2.0 per clk per SM) plus one DADD and
 # one max.f64 (1.7 per clk per SM each), measured on this GB300; nominal 1.25 TFLOP/s FP64.
 FP64_TERMS_PER_CLK_PER_SM = 1.0 / (1.0 / 2.0 + 2.0 / 1.7)

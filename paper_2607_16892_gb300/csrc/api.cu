@@ -20,6 +20,7 @@
 namespace kvdro {
 int64_t hist_slice_samples();
 int64_t expand_tile_positions();
+int64_t scan_tile_bins();
 }  // namespace kvdro
 
 using kvdro::Prec;
@@ -58,7 +59,7 @@ struct kvdro_ctx {
     std::vector<int64_t> off, pair_off, hist_off, N;
     std::vector<int32_t> L, Lin, hist_blocks, exp_blocks;
 
-    Buf sorted, pairs, hist, csum, sumx, meta, errs, in_stage, grid_in, keys, cost64, out_stage, ranks;
+    Buf sorted, pairs, hist, csum, sumx, meta, errs, in_stage, grid_in, keys, cost64, out_stage, ranks, scan_tot;
     void* pin = nullptr;  // pinned host staging
     size_t pin_bytes = 0;
     cudaEvent_t pin_free = nullptr;  // completes when the last copy out of `pin` is done
@@ -235,7 +236,7 @@ int kvdro_destroy(kvdro_ctx* ctx) {
     DeviceGuard g(ctx->device);
     if (ctx->last_stream) cudaStreamSynchronize(ctx->last_stream);
     cudaDeviceSynchronize();
-    for (Buf* b : {&ctx->sorted, &ctx->pairs, &ctx->hist, &ctx->csum, &ctx->sumx, &ctx->meta, &ctx->errs, &ctx->in_stage,
+    for (Buf* b : {&ctx->sorted, &ctx->scan_tot, &ctx->pairs, &ctx->hist, &ctx->csum, &ctx->sumx, &ctx->meta, &ctx->errs, &ctx->in_stage,
                    &ctx->grid_in, &ctx->keys, &ctx->cost64, &ctx->out_stage, &ctx->ranks})
         release(*b);
     if (ctx->pin) cudaFreeHost(ctx->pin);
@@ -306,6 +307,10 @@ int kvdro_load_samples(kvdro_ctx* ctx, int32_t K, const int64_t* offsets, const 
     if ((rc = ensure(ctx, ctx->csum, (size_t)ctx->hist_total * 8))) return rc;
     if ((rc = ensure(ctx, ctx->sumx, (size_t)K * 8))) return rc;
     if ((rc = ensure(ctx, ctx->errs, 2 * sizeof(int32_t)))) return rc;
+    int64_t max_bins = 0;
+    for (int32_t k = 0; k < K; k++) max_bins = std::max<int64_t>(max_bins, (int64_t)L_max[k] + 1);
+    const int64_t scan_tiles = (max_bins + kvdro::scan_tile_bins() - 1) / kvdro::scan_tile_bins();
+    if ((rc = ensure(ctx, ctx->scan_tot, (size_t)K * scan_tiles * 16))) return rc;
     const size_t meta_bytes = (size_t)(K + 1) * 8 * 3 + (size_t)K * 8 + (size_t)K * 4 * 2 + (size_t)(K + 1) * 4 * 2 + 64;
     if ((rc = ensure(ctx, ctx->meta, meta_bytes))) return rc;
 
@@ -356,6 +361,8 @@ int kvdro_load_samples(kvdro_ctx* ctx, int32_t K, const int64_t* offsets, const 
     a.sorted = static_cast<int32_t*>(ctx->sorted.p);
     a.pairs = static_cast<float2*>(ctx->pairs.p);
     a.err = static_cast<int32_t*>(ctx->errs.p);
+    a.tile_tot = static_cast<int64_t*>(ctx->scan_tot.p);
+    a.scan_tiles = (int32_t)scan_tiles;
     a.K = K;
     KV_CUDA(kvdro::launch_histogram(a, ctx->hist_blocks[K], s), "histogram kernel");
     KV_CUDA(kvdro::launch_scan(a, s), "scan kernel");

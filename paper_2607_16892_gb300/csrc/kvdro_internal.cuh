@@ -29,6 +29,8 @@ struct SortArgs {
     int32_t* sorted;            // [offsets[K]]
     float2* pairs;              // [pair_off[K]]
     int32_t* err;               // [0] += out-of-range samples
+    int64_t* tile_tot;          // [K][scan_tiles][2] scan tile totals (count, sum of v h[v])
+    int32_t scan_tiles;         // scan tiles of the largest class: ceil((max L + 1) / scan tile bins)
     int32_t K;
 };
 

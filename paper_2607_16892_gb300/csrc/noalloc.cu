@@ -19,6 +19,7 @@
 namespace kvdro {
 int64_t hist_slice_samples();
 int64_t expand_tile_positions();
+int64_t scan_tile_bins();
 }  // namespace kvdro
 
 namespace {
@@ -121,7 +122,7 @@ extern "C" int kvdro_eval_grid_noalloc(int32_t K, const int64_t* offsets, const 
     if (R < 1 || R > (1 << 20) || NL < 1 || NL > 256 || E < 1 || E > 64 || M < 1 || M > 65536)
         return report(err, err_len, KVDRO_EINVAL, "R, NL, E or M out of range");
     const int64_t slice = kvdro::hist_slice_samples(), tile = kvdro::expand_tile_positions();
-    int64_t pair_total = 0, hist_total = 0, hist_blocks = 0, exp_blocks = 0;
+    int64_t pair_total = 0, hist_total = 0, hist_blocks = 0, exp_blocks = 0, max_bins = 0;
     for (int32_t k = 0; k < K; k++) {
         const int64_t n = offsets[k + 1] - offsets[k];
         const int64_t lin = L_in ? L_in[k] : 0;
@@ -131,6 +132,7 @@ extern "C" int kvdro_eval_grid_noalloc(int32_t K, const int64_t* offsets, const 
         const int64_t padn = (n + kvdro::kPadSamples - 1) / kvdro::kPadSamples * kvdro::kPadSamples;
         pair_total += padn;
         hist_total += (int64_t)L_max[k] + 1;
+        max_bins = max_bins > (int64_t)L_max[k] + 1 ? max_bins : (int64_t)L_max[k] + 1;
         hist_blocks += (n + slice - 1) / slice;
         exp_blocks += (padn + tile - 1) / tile;
     }
@@ -173,6 +175,8 @@ extern "C" int kvdro_eval_grid_noalloc(int32_t K, const int64_t* offsets, const 
     const size_t o_sorted = take((size_t)total * 4);
     const size_t o_pairs = take((size_t)pair_total * 8);
     const size_t o_keys = take((size_t)rows * 8);
+    const int64_t scan_tiles = (max_bins + kvdro::scan_tile_bins() - 1) / kvdro::scan_tile_bins();
+    const size_t o_tiles = take((size_t)K * scan_tiles * 16);
     if (o > (size_t)KVDRO_NOALLOC_SCRATCH_BYTES) {
         char msg[200];
         snprintf(msg, sizeof(msg), "the problem needs %zu bytes of scratch; the static scratch holds %zu bytes", o,
@@ -243,6 +247,8 @@ extern "C" int kvdro_eval_grid_noalloc(int32_t K, const int64_t* offsets, const 
     sa.sorted = reinterpret_cast<int32_t*>(S + o_sorted);
     sa.pairs = reinterpret_cast<float2*>(S + o_pairs);
     sa.err = reinterpret_cast<int32_t*>(S + o_err);
+    sa.tile_tot = reinterpret_cast<int64_t*>(S + o_tiles);
+    sa.scan_tiles = (int32_t)scan_tiles;
     sa.K = K;
     NA_CUDA(kvdro::launch_histogram(sa, (int32_t)hist_blocks, s));
     NA_CUDA(kvdro::launch_scan(sa, s));

@@ -15,9 +15,11 @@ constexpr int kHistThreads = 512;
 constexpr int64_t kHistSlice = 1 << 16;  // samples per histogram block
 constexpr int kHistSmemBins = 16384;     // bins [0, 16384) privatised in shared memory (64 KB)
 constexpr int kScanThreads = 1024;
+constexpr int64_t kScanTile = (int64_t)kScanThreads * 4;  // bins per scan block
 constexpr int kExpandThreads = 512;
 constexpr int kExpandPerThread = 8;
 constexpr int64_t kExpandTile = (int64_t)kExpandThreads * kExpandPerThread;
+constexpr int kExpandCoarse = 2048;  // entries of the per-block coarse index of cumulative counts (8 KB)
 
 __device__ __forceinline__ int find_segment(const int32_t* prefix, int K, int b) {
     // largest k with prefix[k] <= b; prefix is strictly increasing, prefix[0] = 0
@@ -44,13 +46,36 @@ __global__ void __launch_bounds__(kHistThreads) k_histogram(SortArgs a) {
     __syncthreads();
     int bad = 0;
     unsigned long long sum = 0;
-    for (int64_t i = beg + threadIdx.x; i < end; i += blockDim.x) {
-        const int32_t x = __ldg(a.lengths + i);
-        if (x < 0 || x > Lk) { bad++; continue; }
+    auto count = [&](int32_t x) {
+        if (x < 0 || x > Lk) {
+            bad++;
+            return;
+        }
         sum += (unsigned long long)x;
         if (x < nb) atomicAdd(&sh_bins[x], 1);
         else atomicAdd(&gh[x], 1);
+    };
+    // 16-byte loads of four samples over the slice's aligned middle (alignment is taken from the
+    // address: `lengths` is the caller's pointer), two loads in flight per thread per step;
+    // the unaligned head and the tail one sample at a time.
+    const int32_t* src = a.lengths;
+    const int64_t mis = (int64_t)((reinterpret_cast<uintptr_t>(src + beg) >> 2) & 3);
+    const int64_t vbeg = min(end, beg + ((4 - mis) & 3));
+    const int64_t nvec = (end - vbeg) >> 2;
+    const int64_t vend = vbeg + 4 * nvec;
+    for (int64_t i = beg + threadIdx.x; i < vbeg; i += blockDim.x) count(__ldg(src + i));
+    const int4* v4 = reinterpret_cast<const int4*>(src + vbeg);
+    int64_t q = threadIdx.x;
+    for (; q + (int64_t)blockDim.x < nvec; q += 2 * (int64_t)blockDim.x) {
+        const int4 u = __ldg(v4 + q), w = __ldg(v4 + q + blockDim.x);
+        count(u.x); count(u.y); count(u.z); count(u.w);
+        count(w.x); count(w.y); count(w.z); count(w.w);
     }
+    if (q < nvec) {
+        const int4 u = __ldg(v4 + q);
+        count(u.x); count(u.y); count(u.z); count(u.w);
+    }
+    for (int64_t i = vend + threadIdx.x; i < end; i += blockDim.x) count(__ldg(src + i));
     __syncthreads();
     for (int v = threadIdx.x; v < nb; v += blockDim.x) {
         const int c = sh_bins[v];
@@ -101,128 +126,177 @@ __device__ __forceinline__ T block_inclusive_scan(T t, T* warp_tot, T* total) {
     return before;
 }
 
-// Per class (one block): cumulative sums sum_{x <= v} x (if requested), then the in-place
-// inclusive scan of the histogram into cumulative counts.
-__global__ void __launch_bounds__(kScanThreads) k_scan(SortArgs a) {
-    __shared__ int32_t warp_tot[kScanThreads / 32];
-    __shared__ long long warp_tot64[kScanThreads / 32];
-    const int k = blockIdx.x;
-    int32_t* h = a.hist + a.hist_off[k];
-    const int64_t n = (int64_t)a.L[k] + 1;
+// Block-wide sum of one value per thread; every thread gets the total.
+template <typename T>
+__device__ __forceinline__ T block_sum(T t, T* warp_tot) {
+#pragma unroll
+    for (int o = 16; o; o >>= 1) t += __shfl_xor_sync(0xffffffffu, t, o);
     const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
-    if (a.csum) {
-        long long* cs = reinterpret_cast<long long*>(a.csum + a.hist_off[k]);
-        long long carry64 = 0;
-        for (int64_t base = 0; base < n; base += (int64_t)kScanThreads * 4) {
-            const int64_t i0 = base + (int64_t)threadIdx.x * 4;
-            long long v[4], t = 0;
+    if (l == 0) warp_tot[w] = t;
+    __syncthreads();
+    T s = l < (int)(blockDim.x >> 5) ? warp_tot[l] : (T)0;
 #pragma unroll
-            for (int j = 0; j < 4; j++) {
-                v[j] = (i0 + j < n) ? (long long)(i0 + j) * h[i0 + j] : 0;
-                t += v[j];
-                v[j] = t;
-            }
-            long long total;
-            const long long incl = block_inclusive_scan<long long>(t, warp_tot64, &total);
+    for (int o = 16; o; o >>= 1) s += __shfl_xor_sync(0xffffffffu, s, o);
+    __syncthreads();  // warp_tot is reused by the caller
+    return s;
+}
+
+// The cumulative counts (and sums) of every class in two passes over tiles of kScanTile bins,
+// one block per (tile, class) so that every SM takes part: first each tile's count total (and
+// its sum of v h[v]), then each tile's inclusive scan, offset by the totals of the class's
+// earlier tiles.  The counts are scanned in place into C[v] = #{x <= v}; the sums go to
+// csum[v] = sum_{x <= v} x when it is requested.
+__global__ void __launch_bounds__(kScanThreads) k_scan_totals(SortArgs a) {
+    __shared__ long long warp_tot[kScanThreads / 32];
+    const int k = blockIdx.y;
+    const int64_t n = (int64_t)a.L[k] + 1, b0 = (int64_t)blockIdx.x * kScanTile;
+    if (b0 >= n) return;  // the class has fewer tiles
+    const int32_t* h = a.hist + a.hist_off[k];
+    long long c = 0, v = 0;
 #pragma unroll
-            for (int j = 0; j < 4; j++)
-                if (i0 + j < n) cs[i0 + j] = carry64 + incl - t + v[j];
-            carry64 += total;
+    for (int j = 0; j < 4; j++) {
+        const int64_t i = b0 + (int64_t)threadIdx.x * 4 + j;
+        if (i < n) {
+            const long long hi = h[i];
+            c += hi;
+            v += i * hi;
         }
     }
-    int32_t carry = 0;
-    for (int64_t base = 0; base < n; base += (int64_t)kScanThreads * 4) {
-        const int64_t i0 = base + (int64_t)threadIdx.x * 4;
-        int32_t v[4], t = 0;
-#pragma unroll
-        for (int j = 0; j < 4; j++) {
-            v[j] = (i0 + j < n) ? h[i0 + j] : 0;
-            t += v[j];
-            v[j] = t;
-        }
-        int32_t incl = t;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const int32_t y = __shfl_up_sync(0xffffffffu, incl, o);
-            if (l >= o) incl += y;
-        }
-        if (l == 31) warp_tot[w] = incl;
-        __syncthreads();
-        if (w == 0) {
-            int32_t s = warp_tot[l];
-#pragma unroll
-            for (int o = 1; o < 32; o <<= 1) {
-                const int32_t y = __shfl_up_sync(0xffffffffu, s, o);
-                if (l >= o) s += y;
-            }
-            warp_tot[l] = s;  // inclusive prefix of warp totals
-        }
-        __syncthreads();
-        const int32_t before = carry + (w ? warp_tot[w - 1] : 0) + incl - t;
-#pragma unroll
-        for (int j = 0; j < 4; j++)
-            if (i0 + j < n) h[i0 + j] = before + v[j];
-        carry += warp_tot[kScanThreads / 32 - 1];
-        __syncthreads();
+    c = block_sum<long long>(c, warp_tot);
+    if (a.csum) v = block_sum<long long>(v, warp_tot);
+    if (threadIdx.x == 0) {
+        const int64_t o = (int64_t)k * a.scan_tiles + blockIdx.x;
+        a.tile_tot[2 * o] = c;
+        a.tile_tot[2 * o + 1] = v;
     }
 }
 
+__global__ void __launch_bounds__(kScanThreads) k_scan_apply(SortArgs a) {
+    __shared__ long long warp_tot[kScanThreads / 32];
+    __shared__ int32_t warp_tot32[kScanThreads / 32];
+    const int k = blockIdx.y;
+    const int64_t n = (int64_t)a.L[k] + 1, b0 = (int64_t)blockIdx.x * kScanTile;
+    if (b0 >= n) return;
+    int32_t* h = a.hist + a.hist_off[k];
+    // carry-in: the totals of this class's earlier tiles
+    long long cc = 0, cv = 0;
+    for (int u = threadIdx.x; u < (int)blockIdx.x; u += blockDim.x) {
+        const int64_t o = (int64_t)k * a.scan_tiles + u;
+        cc += a.tile_tot[2 * o];
+        cv += a.tile_tot[2 * o + 1];
+    }
+    cc = block_sum<long long>(cc, warp_tot);
+    if (a.csum) cv = block_sum<long long>(cv, warp_tot);
+    const int64_t i0 = b0 + (int64_t)threadIdx.x * 4;
+    int32_t cnt[4];
+#pragma unroll
+    for (int j = 0; j < 4; j++) cnt[j] = (i0 + j < n) ? h[i0 + j] : 0;
+    if (a.csum) {
+        long long* cs = reinterpret_cast<long long*>(a.csum + a.hist_off[k]);
+        long long w[4], t = 0;
+#pragma unroll
+        for (int j = 0; j < 4; j++) {
+            t += (long long)(i0 + j) * cnt[j];
+            w[j] = t;
+        }
+        long long total;
+        const long long incl = block_inclusive_scan<long long>(t, warp_tot, &total);
+#pragma unroll
+        for (int j = 0; j < 4; j++)
+            if (i0 + j < n) cs[i0 + j] = cv + incl - t + w[j];
+    }
+    int32_t w[4], t = 0;
+#pragma unroll
+    for (int j = 0; j < 4; j++) {
+        t += cnt[j];
+        w[j] = t;
+    }
+    int32_t total;
+    const int32_t incl = block_inclusive_scan<int32_t>(t, warp_tot32, &total);
+#pragma unroll
+    for (int j = 0; j < 4; j++)
+        if (i0 + j < n) h[i0 + j] = (int32_t)(cc + incl - t + w[j]);
+}
+
 __global__ void __launch_bounds__(kExpandThreads) k_expand(SortArgs a) {
+    // A coarse index of the class's cumulative counts in shared memory: entry c is C at the end of
+    // bucket c (buckets of `stride` consecutive bins).  Each thread finds its first position's
+    // bucket there, then the bin inside the bucket in global memory (log2(stride) steps), and
+    // walks on for its next positions.  The warp then stores its 256 values lane-contiguously
+    // through shared memory (rows of 9 words: conflict-free), so every store is coalesced.
+    __shared__ int32_t sK[kExpandCoarse];
+    __shared__ int32_t sV[kExpandThreads / 32][32 * 9];
     const int k = find_segment(a.exp_blocks, a.K, blockIdx.x);
     const int64_t tile = blockIdx.x - a.exp_blocks[k];
     const int64_t Nk = a.offsets[k + 1] - a.offsets[k];
     const int64_t padk = a.pair_off[k + 1] - a.pair_off[k];
     const int32_t* C = a.hist + a.hist_off[k];
     const int32_t Lk = a.L[k];
+    const int32_t stride = (int32_t)(((int64_t)Lk + kExpandCoarse) / kExpandCoarse);  // ceil((Lk + 1) / kExpandCoarse)
+    const int32_t ncoarse = (int32_t)(((int64_t)Lk + stride) / stride);                 // ceil((Lk + 1) / stride)
+    for (int c = threadIdx.x; c < ncoarse; c += blockDim.x)
+        sK[c] = __ldg(C + min((int64_t)Lk, (int64_t)(c + 1) * stride - 1));
+    __syncthreads();
+    const int lane = threadIdx.x & 31;
+    int32_t* wv = sV[threadIdx.x >> 5];
     const int64_t p0 = tile * kExpandTile + (int64_t)threadIdx.x * kExpandPerThread;
-    if (p0 >= padk) return;
-    int32_t* out = a.sorted + a.offsets[k];
-    float2* pr = a.pairs + a.pair_off[k];
-    float vals[kExpandPerThread];
     if (p0 < Nk) {
-        // smallest v with C[v] > p0 (C[Lk] = Nk > p0 guarantees existence)
-        int32_t lo = 0, hi = Lk;
+        // smallest bucket c with sK[c] > p0 (the last bucket ends at Lk and C[Lk] = Nk > p0)
+        int32_t lo = 0, hi = ncoarse - 1;
         while (lo < hi) {
             const int32_t mid = (lo + hi) >> 1;
-            if ((int64_t)__ldg(C + mid) > p0) hi = mid; else lo = mid + 1;
+            if ((int64_t)sK[mid] > p0) hi = mid; else lo = mid + 1;
         }
-        int32_t v = lo;
+        // then the smallest v in the bucket with C[v] > p0 (C at the bucket's end is sK[lo] > p0)
+        int32_t a0 = lo * stride, b0 = (int32_t)min((int64_t)Lk, (int64_t)(lo + 1) * stride - 1);
+        while (a0 < b0) {
+            const int32_t mid = (a0 + b0) >> 1;
+            if ((int64_t)__ldg(C + mid) > p0) b0 = mid; else a0 = mid + 1;
+        }
+        int32_t v = a0;
 #pragma unroll
         for (int j = 0; j < kExpandPerThread; j++) {
             const int64_t p = p0 + j;
-            if (p < Nk) {
-                if ((int64_t)__ldg(C + v) <= p) {
-                    // Galloping search for the next bin: doubling steps, then bisection.  Gaps between
-                    // consecutive sorted values can span thousands of empty bins in a heavy tail.
-                    int32_t base = v, step = 1;  // invariant: C[base] <= p
-                    while (step <= Lk - base && (int64_t)__ldg(C + base + step) <= p) {
-                        base += step;
-                        step <<= 1;
-                    }
-                    int32_t a = min(base + 1, Lk), b2 = (step <= Lk - base) ? base + step : Lk;  // both <= Lk
-                    while (a < b2) {
-                        const int32_t mid = (a + b2) >> 1;
-                        if ((int64_t)__ldg(C + mid) > p) b2 = mid; else a = mid + 1;
-                    }
-                    v = a;
+            if (p < Nk && (int64_t)__ldg(C + v) <= p) {
+                // Galloping search for the next bin: doubling steps, then bisection.  Gaps between
+                // consecutive sorted values can span thousands of empty bins in a heavy tail.
+                int32_t base = v, step = 1;  // invariant: C[base] <= p
+                while (step <= Lk - base && (int64_t)__ldg(C + base + step) <= p) {
+                    base += step;
+                    step <<= 1;
                 }
-                out[p] = v;
-                vals[j] = (float)v;
-            } else {
-                vals[j] = __int_as_float(0x7fc00000);  // quiet NaN pad
+                int32_t a = min(base + 1, Lk), b2 = (step <= Lk - base) ? base + step : Lk;  // both <= Lk
+                while (a < b2) {
+                    const int32_t mid = (a + b2) >> 1;
+                    if ((int64_t)__ldg(C + mid) > p) b2 = mid; else a = mid + 1;
+                }
+                v = a;
             }
+            wv[lane * 9 + j] = v;  // positions past Nk are never stored as samples
         }
-    } else {
-#pragma unroll
-        for (int j = 0; j < kExpandPerThread; j++) vals[j] = __int_as_float(0x7fc00000);
     }
-    // p0 is a multiple of 8 and the region starts on a multiple of 128 pairs: 64-byte aligned.
-    float4* dst = reinterpret_cast<float4*>(pr + p0);
+    __syncwarp();
+    // lane-contiguous stores: position idx of the warp's 256 lives at wv[(idx / 8) * 9 + idx % 8]
+    const int64_t wbase = tile * kExpandTile + (int64_t)(threadIdx.x >> 5) * 32 * kExpandPerThread;
+    int32_t* out = a.sorted + a.offsets[k];
+    float2* pr = a.pairs + a.pair_off[k];
 #pragma unroll
-    for (int j = 0; j < kExpandPerThread / 2; j++) {
-        const int64_t p = p0 + 2 * j;
-        if (p + 1 < padk) dst[j] = make_float4(vals[2 * j], vals[2 * j], vals[2 * j + 1], vals[2 * j + 1]);
-        else if (p < padk) pr[p] = make_float2(vals[2 * j], vals[2 * j]);
+    for (int i = 0; i < kExpandPerThread; i++) {
+        const int idx = i * 32 + lane;
+        const int64_t p = wbase + idx;
+        if (p < Nk) out[p] = wv[(idx >> 3) * 9 + (idx & 7)];
+    }
+    const float nan = __int_as_float(0x7fc00000);  // quiet NaN pad
+#pragma unroll
+    for (int i = 0; i < kExpandPerThread / 2; i++) {
+        const int idx = (i * 32 + lane) * 2;  // even: the pair store is 16-byte aligned
+        const int64_t q = wbase + idx;
+        if (q < padk) {
+            const float f0 = q < Nk ? (float)wv[(idx >> 3) * 9 + (idx & 7)] : nan;
+            const float f1 = q + 1 < Nk ? (float)wv[((idx + 1) >> 3) * 9 + ((idx + 1) & 7)] : nan;
+            if (q + 1 < padk) *reinterpret_cast<float4*>(pr + q) = make_float4(f0, f0, f1, f1);
+            else pr[q] = make_float2(f0, f0);
+        }
     }
 }
 
@@ -246,9 +320,15 @@ cudaError_t launch_histogram(const SortArgs& a, int32_t nblocks, cudaStream_t s)
 }
 
 cudaError_t launch_scan(const SortArgs& a, cudaStream_t s) {
-    k_scan<<<a.K, kScanThreads, 0, s>>>(a);
+    const dim3 grid((unsigned)a.scan_tiles, (unsigned)a.K);
+    k_scan_totals<<<grid, kScanThreads, 0, s>>>(a);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    k_scan_apply<<<grid, kScanThreads, 0, s>>>(a);
     return cudaGetLastError();
 }
+
+int64_t scan_tile_bins() { return kScanTile; }
 
 cudaError_t launch_expand(const SortArgs& a, int32_t nblocks, cudaStream_t s) {
     k_expand<<<nblocks, kExpandThreads, 0, s>>>(a);
