@@ -557,7 +557,10 @@ int kvdro_eval_grid(kvdro_ctx* ctx, int precision, int32_t R, const int32_t* r, 
     const int64_t per_m = (int64_t)ctx->K * shape.r_blocks;
     const int64_t m_step = std::max<int64_t>(1, 0x7fffffffLL / per_m);
     ctx->grid_timed = false;
-    if (ctx->skip_chunk >= 0)  // test hook: bounded waits of about 1 ms that run out on one chunk
+    // Test hook: bounded waits of about 1 ms that run out on one chunk.  The setting lives in
+    // device globals, so while it is armed it applies to every grid launch of the process on this
+    // device; only contexts created with KVDRO_TEST_SKIP_CHUNK arm it, around their own launches.
+    if (ctx->skip_chunk >= 0)
         KV_CUDA(kvdro::set_wait_test(ctx->skip_chunk, kTestWaitCycles, s), "arming the wait test");
     KV_CUDA(cudaEventRecord(ctx->grid_t0, s), "recording grid start");
     for (int64_t m0 = 0; m0 < M; m0 += m_step) {
