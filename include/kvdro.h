@@ -67,7 +67,11 @@ typedef enum {
                             FP64 outputs with FP64 rounding only */
 } kvdro_precision;
 
-/* Create a context on CUDA device `device_ordinal`.  *out receives the handle (NULL on error). */
+/* Create a context on CUDA device `device_ordinal`.  *out receives the handle (NULL on error).
+ * Two environment variables, read here, are test hooks and must not be set in production:
+ * KVDRO_TEST_FAIL_ALLOC=n makes the context's n-th allocation fail (KVDRO_ENOMEM), and
+ * KVDRO_TEST_SKIP_CHUNK=c makes the context's grid kernels leave staged chunk c uncopied with a
+ * wait bound of about 1 ms, so every bounded wait on it runs out (KVDRO_ETIMEOUT). */
 int kvdro_create(kvdro_ctx** out, int device_ordinal);
 
 /*
