@@ -59,7 +59,8 @@ struct GridCfg {
     static_assert(P_ == Prec::F64 || TL_ % 2 == 0, "the FP32 and exact tiles pack lam values in pairs");
 };
 // 2 r x 8 lam tiles, up to 16 warps per CTA and (FP32, exact) two CTAs per SM (64 registers)
-// for up to 128 lam values; 2 x 16 tiles for 129..256 lam values.  FP64: 2 x 8 tiles.
+// for up to 128 lam values; for 129..256 lam values the exact kernel runs one CTA of up to 32
+// such warps per SM and the FP32 kernel 2 x 16 tiles.  FP64: 2 x 8 tiles.
 // All stage 4096-sample chunks (32 KB) through a 2-deep ring.  The FP32 variants fold their
 // partial sums every 2 chunks (256 samples per lane); the exact variants fold as often as their
 // support size requires.  The narrow variants unroll the sample loop 8 times.
@@ -67,7 +68,7 @@ using CfgF32 = GridCfg<Prec::F32, 2, 8, 2, 2, 512, 4096, 2, 8>;
 using CfgF32Wide = GridCfg<Prec::F32, 2, 16, 2, 1, 512, 4096, 2, 2>;
 using CfgF64 = GridCfg<Prec::F64, 2, 8, 0, 1, 512, 4096, 2>;
 using CfgExact = GridCfg<Prec::EXACT, 2, 8, 0, 2, 512, 4096, 2, 8>;
-using CfgExactWide = GridCfg<Prec::EXACT, 2, 16, 0, 1, 512, 4096, 2, 4>;
+using CfgExactWide = GridCfg<Prec::EXACT, 2, 8, 0, 1, 1024, 4096, 2, 8>;
 constexpr int kWarpsTarget = 16;  // warps per CTA the r groups fill up to
 
 // ---------------------------------------------------------------- PTX helpers
@@ -447,7 +448,7 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
                 acc[i][jp] = 0ull;
             }
         // Fold the FP32 sums into int64 after `fe` loads of two samples.  Every term is an integer
-        // in [0, L + 2], so a lane's sums stay below 2 fe (L + 2) <= 2^24 and are exact; fe is a
+        // in [0, L + 1], so a lane's sums stay below 2 fe (L + 2) <= 2^24 and are exact; fe is a
         // power of two, the same for every thread of the CTA.
         int fe = 1;
         while (fe < 1024 && 2 * (int64_t)(2 * fe) * (a.L[k] + 2) <= (1ll << 24)) fe <<= 1;
