@@ -255,6 +255,19 @@ def test_exact_mode_rejects_support_above_its_limit():
         kvdro.kvdro_destroy(ctx)
 
 
+@pytest.mark.parametrize("nl", [37, 128, 129, 256])
+def test_fp32_results_are_the_exact_results_rounded(nl):
+    """With every support at most 2^22 an FP32 request runs the exact kernel and rounds its
+    results: S, cost and the minimum cost are the FP64 exact-mode values cast to FP32, bit for bit
+    (lam counts on both sides of the 128 / 256 tile variants)."""
+    w = random_case(21, K=3, N=(3000, 517, 40), L=(4000, 4000, 4000), R=29, n_lam=nl, n_eps=3, M=2,
+                    lam_range=(1e-3, 300.0), eps_max=500.0)
+    f32, ex = run(w, P["fp32"]), run(w, P["exact"])
+    for key in ("S", "cost"):
+        assert np.array_equal(f32[key], ex[key].astype(np.float32)), key
+    compare_full(w, ex, O.solve(w), "exact")
+
+
 @pytest.mark.parametrize("prec", ["exact", "fp32"])
 def test_exact_kernel_at_its_largest_support(prec):
     """L = 2^22, the largest support the exact kernel takes: its FP32 sums fold after every
