@@ -1,7 +1,8 @@
 """GB300 (sm_103a) evaluator of the Wasserstein-DRO KV-reservation cost grid.
 
 The computation lives in the CUDA library built from ``csrc/`` (C ABI in
-``include/kvdro.h``); ``kvdro`` is its Python binding.
+``include/kvdro.h``); ``kvdro`` is its Python binding.  ``bcd`` runs the block-coordinate
+descent of Alg. 1 on the host around the library's worst-case cost curves.
 """
 
 from . import kvdro  # noqa: F401
@@ -15,6 +16,7 @@ from .kvdro import (  # noqa: F401
     kvdro_destroy,
     kvdro_eval_dual,
     kvdro_eval_grid,
+    kvdro_eval_grid_noalloc,
     kvdro_last_error,
     kvdro_last_grid_ms,
     kvdro_load_samples,
