@@ -42,7 +42,7 @@ __device__ __forceinline__ void g_and_slope(const ClassView& c, double eta, doub
     const double mu = fmin(gam, cp), nu = fmin(gam, cw), kap = mu + nu;
     const double dmu = gam < cp ? 1.0 : 0.0, dnu = gam < cw ? 1.0 : 0.0;
     const double L = (double)c.L, N = (double)c.N;
-    const double d = (cp - mu) * L - (cp + cw) * eta;
+    const double d = excess_offset(cp, cw, mu, L, eta);
     int64_t cnt, sum;
     tail(c, first_active(kap, d, c.L), cnt, sum);
     const double tot = N * cw * eta - nu * (double)c.sumx + kap * (double)sum + d * (double)cnt;

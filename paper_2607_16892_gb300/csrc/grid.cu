@@ -306,8 +306,8 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
             kap[jp] = pk(v0 ? (float)(mu0 + fmin(l0, cw)) : 0.f, v1 ? (float)(mu1 + fmin(l1, cw)) : 0.f);
 #pragma unroll
             for (int i = 0; i < TR; i++) {
-                const double d0 = (cp - mu0) * Lk - (cp + cw) * eta[i];
-                const double d1 = (cp - mu1) * Lk - (cp + cw) * eta[i];
+                const double d0 = excess_offset(cp, cw, mu0, Lk, eta[i]);
+                const double d1 = excess_offset(cp, cw, mu1, Lk, eta[i]);
                 dd[i][jp] = pk(v0 && rvalid[i] ? (float)d0 : 0.f, v1 && rvalid[i] ? (float)d1 : 0.f);
                 acc[i][jp] = 0ull;
             }
@@ -373,7 +373,7 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
             kap[j] = v ? mu + fmin(l, cw) : 0.0;
 #pragma unroll
             for (int i = 0; i < TR; i++) {
-                dd[i][j] = (v && rvalid[i]) ? (cp - mu) * Lk - (cp + cw) * eta[i] : 0.0;
+                dd[i][j] = (v && rvalid[i]) ? excess_offset(cp, cw, mu, Lk, eta[i]) : 0.0;
                 acc[i][j] = 0.0;
             }
         }
@@ -435,7 +435,7 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
         const double c_lam = s_lam[c_lj];  // s_lam is padded with zeros to NLpad
         const double c_mu = fmin(c_lam, cp), c_kap = c_mu + fmin(c_lam, cw);
         const double c_eta = c_valid ? (double)a.r[c_ri] - (double)a.L_in[k] : 0.0;
-        const double c_d = (cp - c_mu) * Lk - (cp + cw) * c_eta;
+        const double c_d = excess_offset(cp, cw, c_mu, Lk, c_eta);
         // t = L + 1 means "none" (no sample exceeds L); t in [0, L + 1] keeps |x + 1 - t| <= L + 1
         const float c_t = (float)(c_valid ? first_active(c_kap, c_d, a.L[k]) : (int64_t)a.L[k] + 1);
 #pragma unroll
@@ -597,7 +597,7 @@ __global__ void __launch_bounds__(kEnvThreads) k_envelope(const GridArgs a) {
         const double eta = (double)a.r[ri] - (double)a.L_in[k];
         const double lam = s_lam[j];
         const double mu = fmin(lam, cp), nu = fmin(lam, cw), kap = mu + nu;
-        const double d = (cp - mu) * (double)Lk - (cp + cw) * eta;
+        const double d = excess_offset(cp, cw, mu, (double)Lk, eta);
         const int64_t t = first_active(kap, d, Lk);  // first active sample value, in [0, L + 1]
         const int64_t below_n = t >= 1 ? (int64_t)C[t - 1] : 0;
         const int64_t below_s = t >= 1 ? CS[t - 1] : 0;

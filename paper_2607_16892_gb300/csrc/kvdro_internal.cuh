@@ -130,6 +130,14 @@ cudaError_t launch_dual(const DualArgs& a, cudaStream_t s);
 
 
 #ifdef __CUDACC__
+// The offset d = (c_p - mu) L - (c_p + c_w) eta of a cell's excess kappa x + d, evaluated as
+// c_p (L - eta) - (mu L + c_w eta): L - eta is an exact integer and every product is rounded once,
+// so a large c_p never swallows a small mu or c_w (the first form cancels to 0 at eta = L when
+// mu and c_w are far below c_p, though d is then -(mu + c_w) L).
+__device__ __forceinline__ double excess_offset(double cp, double cw, double mu, double L, double eta) {
+    return cp * (L - eta) - (mu * L + cw * eta);
+}
+
 // The first active support point of a cell: the smallest integer t in [0, L] with
 // kappa * t + d > 0, or L + 1 when there is none (kappa >= 0, so the condition is monotone in
 // t).  One FMA gives the sign of kappa * t + d exactly, so each test is exact.  An FP32 estimate

@@ -255,6 +255,19 @@ def test_exact_mode_rejects_support_above_its_limit():
         kvdro.kvdro_destroy(ctx)
 
 
+@pytest.mark.parametrize("prec", ["exact", "fp64", "envelope"])
+def test_multipliers_and_costs_far_below_fp32_range(prec):
+    """kappa below FP32's smallest normal (the FP32 estimate of a cell's threshold overflows and the
+    FP64 quotient settles it), and c_w or mu many orders below c_p (the excess offset d must not
+    lose them to cancellation).  FP32 outputs cannot hold costs of 1e-248; FP32 requests run the
+    same exact kernel (test_fp32_results_are_the_exact_results_rounded)."""
+    rng = np.random.default_rng(17)
+    w = make([rng.integers(0, 300, 2000), rng.integers(100, 301, 60)], 300, [0, 7, 150, 299, 300],
+             [1e-300, 1e-200, 1e-45, 1e-38, 1e-20, 0.5], [0.0, 1e-10, 3.0], [10.0, 1e-300, 2.0], [1.0, 1e-300, 1e-250])
+    mode = kvdro.KVDRO_ENVELOPE if prec == "envelope" else P[prec]
+    compare_full(w, run(w, mode), O.solve(w), "fp64" if prec == "envelope" else prec)
+
+
 @pytest.mark.parametrize("nl", [37, 128, 129, 256])
 def test_fp32_results_are_the_exact_results_rounded(nl):
     """With every support at most 2^22 an FP32 request runs the exact kernel and rounds its
