@@ -124,8 +124,9 @@ int kvdro_eval_grid(kvdro_ctx* ctx, int precision, int32_t R, const int32_t* r, 
  * eq. app_kantorovich; the value of the epigraph LP of eq. app_lp, which equals the worst case
  * over the Wasserstein ball by the strong duality of App. A Step 2).  The objective is convex
  * and piecewise linear in gamma with its minimiser in [0, max(c_p, c_w)]; the library bisects on
- * its right derivative (64 halvings) with every evaluation O(1) from the sorted samples'
- * cumulative counts and sums, so results carry FP64 rounding only.
+ * its right derivative over the ordered bit patterns of the nonnegative doubles (at most 63
+ * steps, down to two adjacent doubles at any scale) with every evaluation O(1) from the sorted
+ * samples' cumulative counts and sums, so results carry FP64 rounding only.
  * Arguments as kvdro_eval_grid; outputs (each may be NULL; host or device):
  *   cost       double [M][E][K][R]   the exact dual value
  *   gamma      double [M][E][K][R]   a minimising gamma

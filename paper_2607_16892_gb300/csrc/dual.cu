@@ -3,12 +3,14 @@
 // g is convex and piecewise linear in gamma (each sample's supremum is a maximum of lines in
 // gamma).  For gamma >= max(c_p, c_w) moving mass never pays and S is the empirical cost, so g
 // rises with slope eps and the minimiser lies in [0, max(c_p, c_w)].  One thread per
-// (regime, radius, class, reservation) bisects on the sign of the right derivative; every
-// evaluation of S and of its derivative is O(1) from the class's cumulative counts and sums:
-// with mu = min(gamma, c_p), nu = min(gamma, c_w), kappa = mu + nu and
-// d = (c_p - mu) L - (c_p + c_w) eta, the samples with a positive excess kappa x + d are x >= t
-// for an integer threshold t, and
-//   N S = N c_w eta - nu sum(x) + kappa sum_{x >= t} x + d #{x >= t}.
+// (regime, radius, class, reservation) bisects on the sign of the right derivative over the
+// bit patterns of the nonnegative doubles (ordered as their values), so the bracket closes to
+// two adjacent doubles in at most 63 steps at any scale: a kink at c_w = 1e-250 under c_p = 2
+// is found as surely as one near c_p.  Every evaluation of S and of its derivative is O(1) from
+// the class's cumulative counts and sums: with mu = min(gamma, c_p), nu = min(gamma, c_w),
+// kappa = mu + nu and d = (c_p - mu) L - (c_p + c_w) eta, the samples with a positive excess
+// kappa x + d (where U beats V) are x >= t for an integer threshold t, and
+//   N S = c_w eta #{x < t} - nu sum_{x < t} x + c_p (L - eta) #{x >= t} - mu sum_{x >= t} (L - x).
 #include <float.h>
 #include <math.h>
 
@@ -18,7 +20,7 @@ namespace kvdro {
 namespace {
 
 constexpr int kDualThreads = 256;
-constexpr int kBisections = 64;
+constexpr int kBisections = 64;  // > 63: enough to close any bracket [0, hi] to adjacent doubles
 
 struct ClassView {
     const int32_t* C;   // cumulative counts, L + 1 entries
@@ -45,11 +47,11 @@ __device__ __forceinline__ void g_and_slope(const ClassView& c, double eta, doub
     const double d = excess_offset(cp, cw, mu, L, eta);
     int64_t cnt, sum;
     tail(c, first_active(kap, d, c.L), cnt, sum);
-    const double tot = N * cw * eta - nu * (double)c.sumx + kap * (double)sum + d * (double)cnt;
-    g = gam * eps + tot * inv_n;
+    const int64_t below = c.sumx - sum, dist = (int64_t)c.L * cnt - sum;  // sum x below t, sum (L - x) from t on
+    g = gam * eps + branch_sum(cp, cw, mu, nu, L, eta, N, cnt, below, dist) * inv_n;
     // right derivative: the active set just above gamma is the one at gamma up to samples whose
     // excess is exactly zero, which change the value by nothing and the slope only at a kink
-    slope = eps + (-dnu * (double)c.sumx + (dmu + dnu) * (double)sum - dmu * L * (double)cnt) * inv_n;
+    slope = eps - (dnu * (double)below + dmu * (double)dist) * inv_n;
 }
 
 __global__ void __launch_bounds__(kDualThreads) k_dual(const DualArgs a) {
@@ -77,17 +79,29 @@ __global__ void __launch_bounds__(kDualThreads) k_dual(const DualArgs a) {
     double best_g = g_lo, best_gam = lo;
     if (s_lo < 0.0 && hi > 0.0) {
         g_and_slope(c, eta, cp, cw, eps, hi, inv_n, g_hi, s_hi);
-        for (int it = 0; it < kBisections; it++) {
-            const double mid = 0.5 * (lo + hi);
-            if (!(mid > lo && mid < hi)) break;
+        long long lb = __double_as_longlong(lo), hb = __double_as_longlong(hi);  // 0 <= lb < hb < 2^63
+        for (int it = 0; it < kBisections && hb - lb > 1; it++) {
+            const long long mb = lb + (hb - lb) / 2;
+            const double mid = __longlong_as_double(mb);
             double gm, sm;
             g_and_slope(c, eta, cp, cw, eps, mid, inv_n, gm, sm);
-            if (sm >= 0.0) { hi = mid; g_hi = gm; }
-            else { lo = mid; g_lo = gm; }
+            if (sm >= 0.0) { hb = mb; hi = mid; g_hi = gm; }
+            else { lb = mb; lo = mid; g_lo = gm; }
         }
         // g is linear between kinks: the better end of the final bracket is the minimum
         if (g_hi < g_lo) { best_g = g_hi; best_gam = hi; }
         else { best_g = g_lo; best_gam = lo; }
+    }
+    // Every g is at least the empirical cost (1/N) sum Q(eta, x_n): the empirical distribution
+    // lies in the ball, and phi >= Q(eta, x) at every gamma.  That bound is exact from integer
+    // sums, whereas g near a kink sums branches many orders above it when c_p or c_w is extreme;
+    // at eps = 0 it is the value itself.
+    {
+        const int64_t e_i = (int64_t)a.r[ri] - a.L_in[k];  // eta, in [0, L] on the reservation domain
+        int64_t n_up, s_up;
+        tail(c, e_i + 1, n_up, s_up);  // the samples above eta
+        const double emp = (cw * (double)(e_i * (c.N - n_up) - (c.sumx - s_up)) + cp * (double)(s_up - e_i * n_up)) * inv_n;
+        if (best_g < emp) best_g = emp;
     }
     const size_t row = ((size_t)m * a.E + e) * a.K + k;
     if (a.cost) a.cost[row * a.R + ri] = best_g;

@@ -302,13 +302,15 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
             const int j0 = lt * TL + 2 * jp;
             const double l0 = s_lam[j0], l1 = s_lam[j0 + 1];
             const bool v0 = j0 < a.NL, v1 = j0 + 1 < a.NL;
-            const double mu0 = fmin(l0, cp), mu1 = fmin(l1, cp);
-            kap[jp] = pk(v0 ? (float)(mu0 + fmin(l0, cw)) : 0.f, v1 ? (float)(mu1 + fmin(l1, cw)) : 0.f);
+            const double mu0 = fmin(l0, cp), mu1 = fmin(l1, cp), nu0 = fmin(l0, cw), nu1 = fmin(l1, cw);
+            // the split of phi this column sums (see use_u_split): the sign of its excess
+            const float s0 = use_u_split(mu0, nu0) ? -1.f : 1.f, s1 = use_u_split(mu1, nu1) ? -1.f : 1.f;
+            kap[jp] = pk(v0 ? s0 * (float)(mu0 + nu0) : 0.f, v1 ? s1 * (float)(mu1 + nu1) : 0.f);
 #pragma unroll
             for (int i = 0; i < TR; i++) {
                 const double d0 = excess_offset(cp, cw, mu0, Lk, eta[i]);
                 const double d1 = excess_offset(cp, cw, mu1, Lk, eta[i]);
-                dd[i][jp] = pk(v0 && rvalid[i] ? (float)d0 : 0.f, v1 && rvalid[i] ? (float)d1 : 0.f);
+                dd[i][jp] = pk(v0 && rvalid[i] ? s0 * (float)d0 : 0.f, v1 && rvalid[i] ? s1 * (float)d1 : 0.f);
                 acc[i][jp] = 0ull;
             }
         }
@@ -369,11 +371,12 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
             const int lj = lt * TL + j;
             const double l = s_lam[lj];
             const bool v = lj < a.NL;
-            const double mu = fmin(l, cp);
-            kap[j] = v ? mu + fmin(l, cw) : 0.0;
+            const double mu = fmin(l, cp), nu = fmin(l, cw);
+            const double sg = use_u_split(mu, nu) ? -1.0 : 1.0;  // the split of phi this column sums
+            kap[j] = v ? sg * (mu + nu) : 0.0;
 #pragma unroll
             for (int i = 0; i < TR; i++) {
-                dd[i][j] = (v && rvalid[i]) ? excess_offset(cp, cw, mu, Lk, eta[i]) : 0.0;
+                dd[i][j] = (v && rvalid[i]) ? sg * excess_offset(cp, cw, mu, Lk, eta[i]) : 0.0;
                 acc[i][j] = 0.0;
             }
         }
@@ -423,8 +426,8 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
         // integer, exact in FP32) max(y, 0) = (y + |y|) / 2, and sum_n y has a closed form, so each
         // term costs two packed adds: y, then the running sum of |y| (the absolute value rides on
         // the add's operand).  Sums stay integers below 2^24 between folds into int64, hence exact.
-        // The count #{x >= t} comes from the class's cumulative counts; the epilogue forms
-        // kappa * sum + d * count in FP64.
+        // The count #{x >= t} comes from the class's cumulative counts; the epilogue puts every
+        // sample on its branch of phi with these integer sums (branch_sum) in FP64.
         u64 nt[TR][TL / 2], acc[TR][TL / 2];  // nt holds 1 - t per cell
         // Each lane works out the threshold of the cell it owns after the final transposition
         // (cell lane >> (5 - LOG2V)); the warp's V thresholds then reach every lane by shuffles.
@@ -511,8 +514,7 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
         }
         if (!timeout) {
             if (pending > 0) fold();
-            // this lane's cell: the active count from the cumulative counts, then
-            // kappa * sum + d * count in FP64
+            // this lane's cell: the active count from the cumulative counts, then the branch sums
             const long long t = (long long)c_t;  // integer in [0, L + 1]
             const long long Nk = a.N[k];
             const long long count = t <= 0 ? Nk : (t > a.L[k] ? 0 : Nk - (long long)a.cdf[a.hist_off[k] + t - 1]);
@@ -521,9 +523,11 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
             const long long sum_abs = acc_r - npad * (t > 1 ? t - 1 : 1 - t);
             const long long sum_y = a.sumx[k] + Nk * (1 - t);
             const long long sum_relu = (sum_y + sum_abs) / 2;  // each sample adds y + |y| = 2 relu(y)
-            const long long sum = sum_relu + (t - 1) * count;
-            const double kap = c_kap, d = c_d;
-            acc64 = kap * (double)sum + d * (double)count;
+            const long long sum = sum_relu + (t - 1) * count;  // sum_{x >= t} x
+            // each sample on its own branch of phi (exact integer sums): V = c_w eta - nu x below t,
+            // U = c_p (L - eta) - mu (L - x) from t on; no large term cancels another
+            acc64 = branch_sum(cp, cw, c_mu, fmin(c_lam, cw), Lk, c_eta, (double)Nk, count, a.sumx[k] - sum,
+                               (long long)a.L[k] * count - sum);
         }
     }
 
@@ -545,10 +549,21 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
         const int ri = r_cta0 + r_local0 + i, lj = lt * TL + j;
         const bool owner = (lane & ((1 << (5 - LOG2V)) - 1)) == 0;
         if (owner && ri < a.R && lj < a.NL) {
-            const double nu = fmin(s_lam[lj], cw);
+            const double mu = fmin(s_lam[lj], cp), nu = fmin(s_lam[lj], cw);
             const double Nk = (double)a.N[k];
             const double eta_i = (double)a.r[ri] - (double)a.L_in[k];
-            const double tot = Nk * cw * eta_i - nu * (double)a.sumx[k] + acc64;
+            double tot;
+            if constexpr (P == Prec::EXACT) {
+                tot = acc64;  // the branch sums, formed above
+            } else {
+                // the split's base plus its excess sum: sum V + sum max(kappa x + d, 0), or
+                // sum U + sum max(-(kappa x + d), 0)
+                const long long N64 = a.N[k], sx = a.sumx[k];
+                const double base = use_u_split(mu, nu)
+                                        ? cp * (Lk - eta_i) * Nk - mu * (double)((long long)a.L[k] * N64 - sx)
+                                        : cw * eta_i * Nk - nu * (double)sx;
+                tot = base + acc64;
+            }
             const double S = tot / Nk;
             s_S[(r_local0 + i) * NLpad + lj] = S;
             if (a.S_out) {
@@ -587,7 +602,7 @@ __global__ void __launch_bounds__(kEnvThreads) k_envelope(const GridArgs a) {
     const double cp = a.cp[m], cw = a.cw[m];
     const int32_t Lk = a.L[k];
     const int64_t Nk = a.N[k];
-    const double N = (double)Nk, sumx = (double)a.sumx[k], inv_n = 1.0 / N;
+    const double N = (double)Nk, inv_n = 1.0 / N;
     const int32_t* C = a.cdf + a.hist_off[k];
     const int64_t* CS = a.csum + a.hist_off[k];
     for (int cell = threadIdx.x; cell < kEnvR * a.NL; cell += blockDim.x) {
@@ -601,7 +616,8 @@ __global__ void __launch_bounds__(kEnvThreads) k_envelope(const GridArgs a) {
         const int64_t t = first_active(kap, d, Lk);  // first active sample value, in [0, L + 1]
         const int64_t below_n = t >= 1 ? (int64_t)C[t - 1] : 0;
         const int64_t below_s = t >= 1 ? CS[t - 1] : 0;
-        const double tot = N * cw * eta - nu * sumx + kap * (double)(a.sumx[k] - below_s) + d * (double)(Nk - below_n);
+        const int64_t cnt = Nk - below_n, sx = a.sumx[k] - below_s;  // samples from t on, and their sum
+        const double tot = branch_sum(cp, cw, mu, nu, (double)Lk, eta, N, cnt, below_s, (int64_t)Lk * cnt - sx);
         const double S = tot * inv_n;
         s_S[rl * a.NL + j] = S;
         if (a.S_out) static_cast<double*>(a.S_out)[(((size_t)m * a.K + k) * a.R + ri) * a.NL + j] = S;

@@ -133,10 +133,38 @@ cudaError_t launch_dual(const DualArgs& a, cudaStream_t s);
 // The offset d = (c_p - mu) L - (c_p + c_w) eta of a cell's excess kappa x + d, evaluated as
 // c_p (L - eta) - (mu L + c_w eta): L - eta is an exact integer and every product is rounded once,
 // so a large c_p never swallows a small mu or c_w (the first form cancels to 0 at eta = L when
-// mu and c_w are far below c_p, though d is then -(mu + c_w) L).
+// mu and c_w are far below c_p, though d is then -(mu + c_w) L).  At the saturated multiplier
+// mu = c_p the L terms vanish exactly and d = -(c_p + c_w) eta.
 __device__ __forceinline__ double excess_offset(double cp, double cw, double mu, double L, double eta) {
-    return cp * (L - eta) - (mu * L + cw * eta);
+    return mu == cp ? -(cp * eta + cw * eta) : cp * (L - eta) - (mu * L + cw * eta);
 }
+
+// sum_n phi(x_n) with every sample on its own branch: V = c_w eta - nu x for the n - cnt samples
+// below the cell's first active point, U = c_p (L - eta) - mu (L - x) for the cnt samples from it
+// on.  The caller passes exact integer sums: sx_below = sum x below the point, dist_above =
+// sum (L - x) from it on.  Nothing cancels beyond what each branch holds itself, whatever the
+// ratios of c_p, c_w and the multiplier (V + max(U - V, 0) loses everything to cancellation
+// when nu is many orders above the result).
+// c i - m j for integers i, j held exactly in doubles: the rounding error of c i is recovered by
+// one FMA, so the difference is rounded about once however closely the two products agree
+// (forming both products first leaves only their rounding errors when they agree to 16 digits).
+__device__ __forceinline__ double diff_of_products(double c, double i, double m, double j) {
+    const double p = __dmul_rn(c, i);
+    const double e = fma(c, i, -p);  // c i - p exactly, barring underflow
+    return fma(-m, j, p) + e;
+}
+
+__device__ __forceinline__ double branch_sum(double cp, double cw, double mu, double nu, double L, double eta,
+                                             double n, int64_t cnt, int64_t sx_below, int64_t dist_above) {
+    return diff_of_products(cw, eta * (n - (double)cnt), nu, (double)sx_below) +
+           diff_of_products(cp, (L - eta) * (double)cnt, mu, (double)dist_above);
+}
+
+// The per-term kernels sum phi as a base plus excesses: sum V + sum max(U - V, 0), or
+// sum U + sum max(V - U, 0).  Each excess cancels, in the total, against the base's slope term
+// (nu sum x, or mu sum (L - x)) on the samples it covers, so a cell takes the base whose slope
+// is the smaller: U when nu > mu.  U - V = kappa x + d, so the U base negates kappa and d.
+__device__ __forceinline__ bool use_u_split(double mu, double nu) { return nu > mu; }
 
 // The first active support point of a cell: the smallest integer t in [0, L] with
 // kappa * t + d > 0, or L + 1 when there is none (kappa >= 0, so the condition is monotone in

@@ -111,3 +111,74 @@ def test_envelope_mode_lognormal_k8_n1e5_full_grid():
     m = np.zeros(256, np.int64)
     k, r, l = rng.integers(0, w.K, 256), rng.integers(0, len(w.r), 256), rng.integers(0, len(w.lam), 256)
     rel_close(gpu["S"][m, k, r, l], O.eval_cells(w, m, k, r, l), RTOL["fp64"], "S (direct cells)")
+
+
+def exact_empirical_cost(w):
+    """(1/N) sum_n Q(eta, x_n) per [m, k, r], exact (integer sums, c_p and c_w as fractions) and
+    rounded once: the dual's value at eps = 0 and a lower bound at every eps, since the empirical
+    distribution lies in every Wasserstein ball (App. A)."""
+    from fractions import Fraction
+    M, K, R = len(w.cp), w.K, len(w.r)
+    out = np.empty((M, K, R), np.float64)
+    for k in range(K):
+        x = [int(v) for v in w.class_samples(k)]
+        for i in range(R):
+            eta = int(w.r[i]) - int(w.L_in[k])
+            below = sum(eta - v for v in x if v < eta)
+            above = sum(v - eta for v in x if v > eta)
+            for m in range(M):
+                out[m, k, i] = float((Fraction(w.cw[m]) * below + Fraction(w.cp[m]) * above) / len(x))
+    return out
+
+
+def check_dual_scaled(w, gpu, ora):
+    """The dual with c_p and c_w many orders apart.  Its minimiser sits where two of phi's lines
+    cross, lines of size up to c_w eta + c_p (L - eta) + max(c_p, c_w) L; FP64 places a sample at such
+    a crossing only to within eps times that size (the oracle's crossing points as the kernel's
+    thresholds), so a cell compares within rtol plus 16 eps times that size.  The exact bounds hold
+    whatever the scale: cost >= the empirical cost, with equality at eps = 0."""
+    rtol = RTOL["fp64"]
+    M, E, K, R = gpu["cost"].shape
+    cp, cw = np.asarray(w.cp)[:, None, None, None], np.asarray(w.cw)[:, None, None, None]
+    eta = (w.r[None, :].astype(np.float64) - w.L_in[:, None].astype(np.float64))[None, None]  # [1, 1, K, R]
+    L = w.L.astype(np.float64)[None, None, :, None]
+    size = cw * eta + cp * (L - eta) + np.maximum(cp, cw) * L
+    tol = rtol * np.abs(ora["cost"]) + 16 * np.finfo(np.float64).eps * size
+    err = np.abs(gpu["cost"] - ora["cost"])
+    assert np.all(err <= tol), (np.argmax(err - tol), gpu["cost"].ravel()[np.argmax(err - tol)])
+    emp = exact_empirical_cost(w)[:, None]                                       # [M, 1, K, R]
+    assert np.all(gpu["cost"] >= emp * (1 - 4 * np.finfo(np.float64).eps)), "below the empirical cost"
+    at0 = np.asarray(w.eps) == 0.0
+    np.testing.assert_allclose(gpu["cost"][:, at0], np.broadcast_to(emp, gpu["cost"].shape)[:, at0], rtol=4e-15, atol=0)
+    # the chosen reservation is a minimiser within the same tolerance
+    chosen = np.take_along_axis(ora["cost"], gpu["r_idx"][..., None].astype(np.int64), axis=-1)[..., 0]
+    assert np.all(chosen <= ora["cost"].min(axis=-1) + tol.max(axis=-1))
+    np.testing.assert_array_equal(gpu["min_cost"], np.take_along_axis(gpu["cost"], gpu["r_idx"][..., None].astype(np.int64), axis=-1)[..., 0])
+
+
+@pytest.mark.parametrize("scale", ["tiny", "huge"])
+def test_dual_costs_far_outside_fp32_range(scale):
+    """The exact dual with c_w or c_p many orders apart (tiny: down to 1e-300; huge: up to 1e150)."""
+    rng = np.random.default_rng(23)
+    from tests.test_gpu_parity import make
+    if scale == "tiny":
+        w = make([rng.integers(0, 300, 2000), rng.integers(100, 301, 60)], 300, [0, 7, 150, 299, 300], [1.0],
+                 [0.0, 1e-10, 3.0], [10.0, 1e-300, 2.0], [1.0, 1e-300, 1e-250])
+    else:
+        w = make([rng.integers(0, 5000, 1500), rng.integers(4000, 5001, 40)], 5000, [0, 1, 2500, 4999, 5000], [1.0],
+                 [0.0, 1.0, 1e100], [1e150, 1.0, 2e150], [1.0, 1e150, 5e149])
+    check_dual_scaled(w, run_dual(w), O.solve_dual(w))
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_dual_equals_the_empirical_cost_at_eps_zero(seed):
+    """At eps = 0 the worst case over the ball is the empirical cost itself (App. A), for any costs."""
+    rng = np.random.default_rng(300 + seed)
+    w = random_case(300 + seed, K=3, N=(int(rng.integers(1, 3000)), 57, 1), L=(1000, 4096, 300), R=17, n_lam=4,
+                    n_eps=3, M=3, lam_range=(1e-3, 200.0), eps_max=50.0)
+    w.eps[0] = 0.0
+    gpu = run_dual(w)
+    emp = exact_empirical_cost(w)
+    np.testing.assert_allclose(gpu["cost"][:, 0], emp, rtol=4e-15, atol=0)  # a few roundings
+    assert np.all(gpu["cost"] >= emp[:, None] * (1 - 4 * np.finfo(np.float64).eps))
+

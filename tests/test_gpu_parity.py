@@ -268,6 +268,16 @@ def test_multipliers_and_costs_far_below_fp32_range(prec):
     compare_full(w, run(w, mode), O.solve(w), "fp64" if prec == "envelope" else prec)
 
 
+@pytest.mark.parametrize("prec", ["exact", "fp64", "envelope"])
+def test_multipliers_costs_and_radii_far_above_fp32_range(prec):
+    """Costs, multipliers and radii around 1e150 (their products near 1e250 stay finite in FP64)."""
+    rng = np.random.default_rng(19)
+    w = make([rng.integers(0, 5000, 1500), rng.integers(4000, 5001, 40)], 5000, [0, 1, 2500, 4999, 5000],
+             [1e-3, 1.0, 1e120, 1e150, 3e150], [0.0, 1.0, 1e100], [1e150, 1.0, 2e150], [1.0, 1e150, 5e149])
+    mode = kvdro.KVDRO_ENVELOPE if prec == "envelope" else P[prec]
+    compare_full(w, run(w, mode), O.solve(w), "fp64" if prec == "envelope" else prec)
+
+
 @pytest.mark.parametrize("nl", [37, 128, 129, 256])
 def test_fp32_results_are_the_exact_results_rounded(nl):
     """With every support at most 2^22 an FP32 request runs the exact kernel and rounds its
