@@ -39,15 +39,16 @@ from synth import lognormal_workload_k8_n1e5, slice_workload  # noqa: E402
 METRIC = "DRO cost terms/sec (class×r×λ×sample) on 1 GB300; % of FP32/HBM roofline"
 UNIT = "terms/s"
 SM_MAX_MHZ_RECIPE = 2070.0
-# FP32-lane bound of the per-term work: every term needs at least two FP32 lane-operations -- the
-# add (or multiply-add) that forms its excess and the add into the running sum -- and an SM has
-# 128 FP32 lanes, so at most 64 terms per clock per SM.  The remaining operation of a term, the
-# max with zero, runs on the ALU pipe or rides on the add as an absolute value (exact kernel);
-# instruction issue (one per scheduler per clock, two instructions per 32 terms) gives the same
-# 64.  Measured on this GB300: packed f32x2 adds alone reach 127.9 FP32 lane-ops/clk/SM.
-LANE_OPS_PER_CLK_PER_SM = 128.0
-LANE_OPS_PER_TERM = 2.0
-TERMS_PER_CLK_PER_SM = LANE_OPS_PER_CLK_PER_SM / LANE_OPS_PER_TERM
+# Bound of the exact kernel's per-term work.  A term costs one instruction-lane on one of two
+# pipes: packed f32x2 adds on the FMA pipe (128 FP32 lanes/clk/SM, two lane-operations per term:
+# 64 terms/clk/SM) or an integer absolute-difference-and-add (sad) on the ALU pipe (64 lanes/clk/SM,
+# one per term: 64 terms/clk/SM).  The kernel splits every warp's cells between the two, so at
+# most 128 terms per clock per SM, which is also the issue limit (4 schedulers x 1 instruction per
+# clock x 32 lanes, one instruction per term and lane).  Measured on this GB300: packed f32x2 adds
+# alone 127.9 FP32 lane-ops/clk/SM, sad.s32 alone 63.4 terms/clk/SM.
+FMA_TERMS_PER_CLK_PER_SM = 128.0 / 2.0
+ALU_TERMS_PER_CLK_PER_SM = 64.0
+TERMS_PER_CLK_PER_SM = FMA_TERMS_PER_CLK_PER_SM + ALU_TERMS_PER_CLK_PER_SM
 GRID_SOURCE = os.path.join(ROOT, "paper_2607_16892_gb300", "csrc", "grid.cu")
 PROFILE = os.path.join(ROOT, "profiles", "k_grid_exact_lognormal_k8_n1e5.md")
 LAUNCHES_PER_STEP = 7  # histogram, scan totals, scan, expand, quantile gather, grid, argmin finalise
@@ -293,8 +294,8 @@ def run_ours(args):
     roofline = {"bound": "alu", "achieved": achieved, "peak": peak, "unit": UNIT, "frac": achieved / peak,
                 "traffic": profile_traffic(), "kernel": "k_grid<EXACT> (FP32 outputs)",
                 "kernel_ms_mean": kernel_ms,
-                "peak_basis": f"{props.multi_processor_count} SMs x {LANE_OPS_PER_CLK_PER_SM:.0f} FP32 lanes/clk/SM "
-                              f"/ {LANE_OPS_PER_TERM:.0f} FP32 lane-ops per term x {SM_MAX_MHZ_RECIPE:.0f} MHz"}
+                "peak_basis": f"{props.multi_processor_count} SMs x ({FMA_TERMS_PER_CLK_PER_SM:.0f} terms/clk/SM on packed "
+                              f"FP32 adds + {ALU_TERMS_PER_CLK_PER_SM:.0f} on integer sad) x {SM_MAX_MHZ_RECIPE:.0f} MHz"}
     if clocks.get("sm_mhz"):
         roofline["frac_at_sampled_clock"] = achieved / (peak * clocks["sm_mhz"] / SM_MAX_MHZ_RECIPE)
 

@@ -81,6 +81,14 @@ __device__ __forceinline__ u64 pk(float lo, float hi) {
 __device__ __forceinline__ void upk(u64 r, float& lo, float& hi) {
     asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(r));
 }
+__device__ __forceinline__ u64 pki(unsigned lo, unsigned hi) {
+    u64 r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "r"(lo), "r"(hi));
+    return r;
+}
+__device__ __forceinline__ void upki(u64 r, unsigned& lo, unsigned& hi) {
+    asm("mov.b64 {%0, %1}, %2;" : "=r"(lo), "=r"(hi) : "l"(r));
+}
 __device__ __forceinline__ u64 ffma2(u64 a, u64 b, u64 c) {
     u64 r;
     asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
@@ -296,6 +304,8 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
     double acc64 = 0.0;  // this lane's cell after the warp transposition
 
     if constexpr (P == Prec::F32) {
+        const float off = stage_offset(a.L[k]);
+        const u64 noff = pk(-off, -off);  // the staged samples carry the class's offset
         u64 kap[TL / 2], dd[TR][TL / 2], acc[TR][TL / 2];
 #pragma unroll
         for (int jp = 0; jp < TL / 2; jp++) {
@@ -323,8 +333,8 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
                 const int nq = cnt >> 6;  // float4 (two samples) per lane
 #pragma unroll(C::UNROLL)
                 for (int t = 0; t < nq; t++) {
-                    const float4 v = q[lane + 32 * t];
-                    const u64 xa = pk(v.x, v.y), xb = pk(v.z, v.w);
+                    const float4 v = q[lane + 32 * t];  // (x', x') pairs of two samples
+                    const u64 xa = fadd2(pk(v.x, v.y), noff), xb = fadd2(pk(v.z, v.w), noff);
                     // The two samples' excesses are added to each other before they join the running
                     // sum: the same number of adds, half as many additions into the long sum.
 #pragma unroll
@@ -365,6 +375,7 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
             }
         }
     } else if constexpr (P == Prec::F64) {
+        const double offd = (double)stage_offset(a.L[k]);  // the staged samples carry the class's offset
         double kap[TL], dd[TR][TL], acc[TR][TL];
 #pragma unroll
         for (int j = 0; j < TL; j++) {
@@ -389,7 +400,7 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
                 const int nq = cnt >> 6;
                 for (int t = 0; t < nq; t++) {
                     const float4 v = q[lane + 32 * t];
-                    const double xa = (double)v.x, xb = (double)v.z;
+                    const double xa = (double)v.x - offd, xb = (double)v.z - offd;  // exact
 #pragma unroll
                     for (int i = 0; i < TR; i++)
 #pragma unroll
@@ -422,13 +433,23 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
         }
     } else {
         // EXACT: per cell (i, j) the active samples are x >= t_ij for an integer threshold t_ij, and
-        // sum_n max(kappa x_n + d, 0) = kappa sum_{x >= t} x + d #{x >= t}.  With y = x + 1 - t (an
-        // integer, exact in FP32) max(y, 0) = (y + |y|) / 2, and sum_n y has a closed form, so each
-        // term costs two packed adds: y, then the running sum of |y| (the absolute value rides on
-        // the add's operand).  Sums stay integers below 2^24 between folds into int64, hence exact.
-        // The count #{x >= t} comes from the class's cumulative counts; the epilogue puts every
-        // sample on its branch of phi with these integer sums (branch_sum) in FP64.
-        u64 nt[TR][TL / 2], acc[TR][TL / 2];  // nt holds 1 - t per cell
+        // sum_n max(kappa x_n + d, 0) = kappa sum_{x >= t} x + d #{x >= t}.  With c = t - 1,
+        // max(x - c, 0) = (x - c + |x - c|) / 2 and sum_n (x - c) has a closed form, so the kernel
+        // streams sum_n |x - c| only, on two pipes at once.  For half of a warp's lam columns one
+        // packed FP32 add forms y = x' + (1 - t - 2^23) = x - c for two cells and one adds |y| into
+        // the running sum (the absolute value rides on the add's operand); for the other half one
+        // integer absolute-difference-and-add (__sad) works on the staged float's bit pattern,
+        // 0x4B000000 + x.  The two kinds alternate in the instruction stream.  Every value is an
+        // integer below 2^24, so both are exact.  Sums are folded into int64 through the warp
+        // transposition before an FP32 sum could pass 2^24.  The count #{x >= t} comes from the
+        // class's cumulative counts; the epilogue puts every sample on its branch of phi with these
+        // integer sums (branch_sum) in FP64.
+        constexpr int TLF = TL / 2;  // lam columns per r row on the packed FP32 adds (in pairs)
+        constexpr int TLI = TL - TLF;  // lam columns per r row on the integer path
+        static_assert(TLF % 2 == 0 && TLI == TLF, "pairs of packed columns alternate with pairs of integer ones");
+        u64 ntf[TR][TLF / 2], accf[TR][TLF / 2];  // ntf: 1 - t - 2^23 for a pair of cells
+        int cci[TR][TLI];                          // 0x4B000000 + t - 1 per cell
+        unsigned acci[TR][TLI];
         // Each lane works out the threshold of the cell it owns after the final transposition
         // (cell lane >> (5 - LOG2V)); the warp's V thresholds then reach every lane by shuffles.
         const int cidx = lane >> (5 - LOG2V);
@@ -439,37 +460,84 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
         const double c_mu = fmin(c_lam, cp), c_kap = c_mu + fmin(c_lam, cw);
         const double c_eta = c_valid ? (double)a.r[c_ri] - (double)a.L_in[k] : 0.0;
         const double c_d = excess_offset(cp, cw, c_mu, Lk, c_eta);
-        // t = L + 1 means "none" (no sample exceeds L); t in [0, L + 1] keeps |x + 1 - t| <= L + 1
-        const float c_t = (float)(c_valid ? first_active(c_kap, c_d, a.L[k]) : (int64_t)a.L[k] + 1);
+        // t = L + 1 means "none" (no sample exceeds L); t in [0, L + 1] keeps |x - c| <= L + 1
+        const int c_t = (int)(c_valid ? first_active(c_kap, c_d, a.L[k]) : (int64_t)a.L[k] + 1);
 #pragma unroll
-        for (int i = 0; i < TR; i++)
+        for (int i = 0; i < TR; i++) {
 #pragma unroll
-            for (int jp = 0; jp < TL / 2; jp++) {
-                const float t0 = __shfl_sync(0xffffffffu, c_t, (i * TL + 2 * jp) << (5 - LOG2V));
-                const float t1 = __shfl_sync(0xffffffffu, c_t, (i * TL + 2 * jp + 1) << (5 - LOG2V));
-                nt[i][jp] = pk(1.0f - t0, 1.0f - t1);
-                acc[i][jp] = 0ull;
+            for (int jp = 0; jp < TLF / 2; jp++) {
+                const int t0 = __shfl_sync(0xffffffffu, c_t, (i * TL + 2 * jp) << (5 - LOG2V));
+                const int t1 = __shfl_sync(0xffffffffu, c_t, (i * TL + 2 * jp + 1) << (5 - LOG2V));
+                ntf[i][jp] = pk((float)(1 - t0 - (1 << 23)), (float)(1 - t1 - (1 << 23)));  // exact: below 2^24
+                accf[i][jp] = 0ull;
             }
-        // Fold the FP32 sums into int64 after `fe` loads of two samples.  Every term is an integer
-        // in [0, L + 1], so a lane's sums stay below 2 fe (L + 2) <= 2^24 and are exact; fe is a
-        // power of two, the same for every thread of the CTA.
+#pragma unroll
+            for (int jj = 0; jj < TLI; jj++) {
+                cci[i][jj] = kStageBits - 1 + __shfl_sync(0xffffffffu, c_t, (i * TL + TLF + jj) << (5 - LOG2V));
+                acci[i][jj] = 0u;
+            }
+        }
+        // Fold after `fe` loads of two samples: a lane's sums are then at most 2 fe (L + 1) <= 2^24,
+        // exact in FP32, and the transposition's 32-lane sums stay below 2^29; fe is a power of two,
+        // the same for every thread of the CTA.
         int fe = 1;
-        while (fe < 1024 && 2 * (int64_t)(2 * fe) * (a.L[k] + 2) <= (1ll << 24)) fe <<= 1;
+        while (fe < (1 << 20) && 2ll * (2 * fe) * ((int64_t)a.L[k] + 1) <= (1ll << 24)) fe <<= 1;
         long long acc_r = 0;
         auto fold = [&]() {
-            int vs[V];
+            unsigned vs[V];
+#pragma unroll
+            for (int i = 0; i < TR; i++) {
+#pragma unroll
+                for (int jp = 0; jp < TLF / 2; jp++) {
+                    float a0, a1;
+                    upk(accf[i][jp], a0, a1);
+                    vs[i * TL + 2 * jp] = __float2uint_rn(a0);
+                    vs[i * TL + 2 * jp + 1] = __float2uint_rn(a1);
+                    accf[i][jp] = 0ull;
+                }
+#pragma unroll
+                for (int jj = 0; jj < TLI; jj++) {
+                    vs[i * TL + TLF + jj] = acci[i][jj];
+                    acci[i][jj] = 0u;
+                }
+            }
+            acc_r += (long long)transpose_reduce<unsigned, V>(vs, lane);
+        };
+        // one load: two samples' (x', x') pairs into every cell's sum; a pair of packed columns
+        // alternates with a pair of integer columns, add for add
+        auto step = [&](const float4 v) {
+            const u64 xa = pk(v.x, v.y), xb = pk(v.z, v.w);
+            const int ba = __float_as_int(v.x), bb = __float_as_int(v.z);  // 0x4B000000 + x
 #pragma unroll
             for (int i = 0; i < TR; i++)
 #pragma unroll
-                for (int jp = 0; jp < TL / 2; jp++) {
-                    float a0, a1;
-                    upk(acc[i][jp], a0, a1);
-                    vs[i * TL + 2 * jp] = __float2int_rn(a0);
-                    vs[i * TL + 2 * jp + 1] = __float2int_rn(a1);
-                    acc[i][jp] = 0ull;
+                for (int p = 0; p < TLF / 2; p++) {
+                    const int j0 = 2 * p, j1 = 2 * p + 1;
+                    const u64 ya = fadd2(xa, ntf[i][p]);
+                    acci[i][j0] = __sad(ba, cci[i][j0], acci[i][j0]);
+                    const u64 yb = fadd2(xb, ntf[i][p]);
+                    acci[i][j1] = __sad(ba, cci[i][j1], acci[i][j1]);
+                    const u64 sy = fadd2(abs2(ya), abs2(yb));
+                    acci[i][j0] = __sad(bb, cci[i][j0], acci[i][j0]);
+                    accf[i][p] = fadd2(accf[i][p], sy);
+                    acci[i][j1] = __sad(bb, cci[i][j1], acci[i][j1]);
                 }
-            acc_r += (long long)transpose_reduce<int, V>(vs, lane);
         };
+        auto run = [&](const float4* q, int t0, int t1, bool clamp) {
+            if (clamp) {
+#pragma unroll 1
+                for (int t = t0; t < t1; t++) {
+                    float4 v = q[lane + 32 * t];  // NaN padding -> x = 0 (x' = 2^23)
+                    v.x = fmaxf(v.x, kStageOffset), v.y = fmaxf(v.y, kStageOffset);
+                    v.z = fmaxf(v.z, kStageOffset), v.w = fmaxf(v.w, kStageOffset);
+                    step(v);
+                }
+            } else {
+#pragma unroll(C::UNROLL)
+                for (int t = t0; t < t1; t++) step(q[lane + 32 * t]);
+            }
+        };
+        const int64_t n_k = a.N[k];
         int pending = 0;  // loads since the last fold
         for (int c = 0; c < nchunks; c++) {
             const int s = c % C::STAGES;
@@ -478,20 +546,15 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
                 const int cnt = (int)min((int64_t)C::CHUNK, np - (int64_t)c * C::CHUNK);
                 const float4* q = reinterpret_cast<const float4*>(ring + (size_t)s * C::CHUNK);
                 const int nq = cnt >> 6;
+                // loads [0, t_clean) hold samples only; the class's last ones may hold NaN padding,
+                // which they read as x = 0 (x' = 2^23)
+                const int64_t left = n_k - (int64_t)c * C::CHUNK;
+                const int t_clean = left <= 0 ? 0 : (int)min((int64_t)nq, left >> 6);
                 for (int t0 = 0; t0 < nq; t0 += fe) {
                     const int t1 = min(nq, t0 + fe);
-#pragma unroll(C::UNROLL)
-                    for (int t = t0; t < t1; t++) {
-                        const float4 v = q[lane + 32 * t];
-                        const float x0 = relu(v.x), x1 = relu(v.z);  // padding samples (NaN) become 0
-                        const u64 xa = pk(x0, x0), xb = pk(x1, x1);
-#pragma unroll
-                        for (int i = 0; i < TR; i++)
-#pragma unroll
-                            for (int jp = 0; jp < TL / 2; jp++) {
-                                acc[i][jp] = fadd2(acc[i][jp], fadd2(abs2(fadd2(xa, nt[i][jp])), abs2(fadd2(xb, nt[i][jp]))));
-                            }
-                    }
+                    const int tm = max(t0, min(t1, t_clean));
+                    run(q, t0, tm, false);
+                    if (tm < t1) run(q, tm, t1, true);
                     pending += t1 - t0;
                     if (pending >= fe) {
                         fold();
@@ -518,7 +581,8 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
             const long long t = (long long)c_t;  // integer in [0, L + 1]
             const long long Nk = a.N[k];
             const long long count = t <= 0 ? Nk : (t > a.L[k] ? 0 : Nk - (long long)a.cdf[a.hist_off[k] + t - 1]);
-            // acc_r = sum |x + 1 - t| over the samples and the padding zeros; relu = (y + |y|) / 2
+            // acc_r = sum |x - c| over the samples and the padding zeros; with y = x - c,
+            // max(y, 0) = (y + |y|) / 2
             const long long npad = np - Nk;
             const long long sum_abs = acc_r - npad * (t > 1 ? t - 1 : 1 - t);
             const long long sum_y = a.sumx[k] + Nk * (1 - t);

@@ -6,10 +6,12 @@
 
 namespace kvdro {
 
-// Samples of one class are staged for the grid kernel as (x, x) float pairs so that one
-// 128-bit shared-memory load yields the packed operands of two samples.  Each class region
-// starts on a multiple of kPadSamples and is padded with NaN pairs, which contribute exactly
-// zero to the excess sum (max(NaN, 0) = 0 in PTX max.f32 / max.f64).
+// Samples of one class are staged for the grid kernel as (x', x') float pairs, x' the sample plus
+// the class's staging offset (stage_offset below), so that one 128-bit shared-memory load yields
+// the packed operands of two samples.  Each class region starts on a multiple of kPadSamples and
+// is padded with NaN pairs, which contribute exactly zero to the per-term kernels' excess sums
+// (max(NaN, 0) = 0 in PTX max.f32 / max.f64); the exact kernel reads the padding as x = 0 and
+// subtracts its known |0 - c| per cell.
 constexpr int kPadSamples = 128;
 
 // Error bits reported by kernels in ctx->d_err[1].
@@ -41,14 +43,24 @@ cudaError_t launch_expand(const SortArgs& a, int32_t nblocks, cudaStream_t s);
 cudaError_t launch_gather_quantiles(const int32_t* sorted, const int64_t* offsets, const int32_t* rank, int32_t K,
                                     int32_t F, int32_t* out, cudaStream_t s);
 
-// F32: per-term FP32 excess sums folded into FP64.  F64: per-term FP64.  EXACT: per-term FP32
-// threshold decisions with exact integer count and sample-sum accumulation, combined in FP64.
+// F32: per-term FP32 excess sums folded into FP64.  F64: per-term FP64.  EXACT: an exact integer
+// threshold per cell, then per term an exact sum of |x - c| (packed FP32 adds and integer
+// absolute differences side by side on two pipes), combined in FP64.
 // ENVELOPE: the same sums in O(1) per cell from cumulative counts and sums (not per term).
 enum class Prec { F32 = 0, F64 = 1, EXACT = 2, ENVELOPE = 3 };
 constexpr int32_t kExactMaxL = 1 << 22;  // the exact kernel's integer sums need L <= 2^22
 
+// Samples of a class whose support is at most kExactMaxL are staged as x + 2^23.  On [2^23, 2^24)
+// a float's bit pattern is 0x4B000000 + x exactly, so the staged float serves both halves of the
+// exact kernel without a conversion: packed FP32 adds on the value, integer absolute differences
+// on the bits.  Larger supports are staged as x.  The FP32 and FP64 per-term kernels subtract
+// the class's offset (exactly) from every sample.
+constexpr float kStageOffset = 8388608.0f;  // 2^23
+constexpr int32_t kStageBits = 0x4B000000;  // bit pattern of 2^23
+__host__ __device__ inline float stage_offset(int32_t L) { return L <= kExactMaxL ? kStageOffset : 0.0f; }
+
 struct GridArgs {
-    const float2* pairs;        // padded (x, x) pairs
+    const float2* pairs;        // padded (x', x') pairs, x' = x + stage_offset(L_k)
     const int64_t* pair_off;    // [K+1]
     const int64_t* N;           // [K]
     const int64_t* sumx;        // [K]

@@ -2,8 +2,9 @@
 // quantile gather.  The samples are their own sort keys and are bounded by L_k, so class k's
 // sorted order is fully determined by its histogram over [0, L_k]: histogram -> inclusive scan
 // (the cumulative count C[v] = #{x <= v}, i.e. N times the empirical CDF) -> expansion of every
-// output position p into the smallest v with C[v] > p.  The expansion also writes the (x, x)
-// float pairs that the grid kernel streams, NaN-padded to a multiple of kPadSamples per class.
+// output position p into the smallest v with C[v] > p.  The expansion also writes the (x', x')
+// float pairs that the grid kernel streams (x' = x plus the class's staging offset), NaN-padded
+// to a multiple of kPadSamples per class.
 #include <math.h>
 
 #include "kvdro_internal.cuh"
@@ -287,13 +288,14 @@ __global__ void __launch_bounds__(kExpandThreads) k_expand(SortArgs a) {
         if (p < Nk) out[p] = wv[(idx >> 3) * 9 + (idx & 7)];
     }
     const float nan = __int_as_float(0x7fc00000);  // quiet NaN pad
+    const float off = stage_offset(Lk);              // x + 2^23 is exact for L <= 2^22
 #pragma unroll
     for (int i = 0; i < kExpandPerThread / 2; i++) {
         const int idx = (i * 32 + lane) * 2;  // even: the pair store is 16-byte aligned
         const int64_t q = wbase + idx;
         if (q < padk) {
-            const float f0 = q < Nk ? (float)wv[(idx >> 3) * 9 + (idx & 7)] : nan;
-            const float f1 = q + 1 < Nk ? (float)wv[((idx + 1) >> 3) * 9 + ((idx + 1) & 7)] : nan;
+            const float f0 = q < Nk ? (float)wv[(idx >> 3) * 9 + (idx & 7)] + off : nan;
+            const float f1 = q + 1 < Nk ? (float)wv[((idx + 1) >> 3) * 9 + ((idx + 1) & 7)] + off : nan;
             if (q + 1 < padk) *reinterpret_cast<float4*>(pr + q) = make_float4(f0, f0, f1, f1);
             else pr[q] = make_float2(f0, f0);
         }
