@@ -39,19 +39,35 @@ __device__ __forceinline__ void tail(const ClassView& c, int64_t t, int64_t& cnt
 }
 
 // g(gamma) and its right derivative.
-__device__ __forceinline__ void g_and_slope(const ClassView& c, double eta, double cp, double cw, double eps, double gam,
-                                            double inv_n, double& g, double& slope) {
-    const double mu = fmin(gam, cp), nu = fmin(gam, cw), kap = mu + nu;
-    const double dmu = gam < cp ? 1.0 : 0.0, dnu = gam < cw ? 1.0 : 0.0;
-    const double L = (double)c.L, N = (double)c.N;
-    const double d = excess_offset(cp, cw, mu, L, eta);
+// The samples from the first active point t on, where U beats V: their count and sum.
+__device__ __forceinline__ void split_at(const ClassView& c, double eta, double cp, double cw, double gam, double& mu,
+                                         double& nu, int64_t& cnt, int64_t& sum) {
+    mu = fmin(gam, cp);
+    nu = fmin(gam, cw);
+    tail(c, first_active(mu + nu, excess_offset(cp, cw, mu, (double)c.L, eta), c.L), cnt, sum);
+}
+
+// Right derivative of g at gamma: the active set just above gamma is the one at gamma up to
+// samples whose excess is exactly zero, which change the value by nothing and the slope only at
+// a kink.  Only its sign steers the bisection.
+__device__ __forceinline__ double slope_at(const ClassView& c, double eta, double cp, double cw, double eps,
+                                           double gam, double inv_n) {
+    double mu, nu;
     int64_t cnt, sum;
-    tail(c, first_active(kap, d, c.L), cnt, sum);
+    split_at(c, eta, cp, cw, gam, mu, nu, cnt, sum);
+    const double dmu = gam < cp ? 1.0 : 0.0, dnu = gam < cw ? 1.0 : 0.0;
     const int64_t below = c.sumx - sum, dist = (int64_t)c.L * cnt - sum;  // sum x below t, sum (L - x) from t on
-    g = gam * eps + branch_sum(cp, cw, mu, nu, L, eta, N, cnt, below, dist) * inv_n;
-    // right derivative: the active set just above gamma is the one at gamma up to samples whose
-    // excess is exactly zero, which change the value by nothing and the slope only at a kink
-    slope = eps - (dnu * (double)below + dmu * (double)dist) * inv_n;
+    return eps - (dnu * (double)below + dmu * (double)dist) * inv_n;
+}
+
+// g(gamma) = gamma eps + S(eta, gamma), every sample on its own branch of phi.
+__device__ __forceinline__ double value_at(const ClassView& c, double eta, double cp, double cw, double eps,
+                                           double gam, double inv_n) {
+    double mu, nu;
+    int64_t cnt, sum;
+    split_at(c, eta, cp, cw, gam, mu, nu, cnt, sum);
+    const int64_t below = c.sumx - sum, dist = (int64_t)c.L * cnt - sum;
+    return gam * eps + branch_sum(cp, cw, mu, nu, (double)c.L, eta, (double)c.N, cnt, below, dist) * inv_n;
 }
 
 __global__ void __launch_bounds__(kDualThreads) k_dual(const DualArgs a) {
@@ -74,23 +90,23 @@ __global__ void __launch_bounds__(kDualThreads) k_dual(const DualArgs a) {
     const double cp = a.cp[m], cw = a.cw[m], eps = a.eps[e];
     const double eta = (double)a.r[ri] - (double)a.L_in[k];
     const double inv_n = 1.0 / (double)c.N;
-    double lo = 0.0, hi = fmax(cp, cw), g_lo, s_lo, g_hi, s_hi;
-    g_and_slope(c, eta, cp, cw, eps, lo, inv_n, g_lo, s_lo);
-    double best_g = g_lo, best_gam = lo;
-    if (s_lo < 0.0 && hi > 0.0) {
-        g_and_slope(c, eta, cp, cw, eps, hi, inv_n, g_hi, s_hi);
+    double lo = 0.0, hi = fmax(cp, cw);
+    double best_g, best_gam;
+    if (slope_at(c, eta, cp, cw, eps, lo, inv_n) < 0.0 && hi > 0.0) {
         long long lb = __double_as_longlong(lo), hb = __double_as_longlong(hi);  // 0 <= lb < hb < 2^63
         for (int it = 0; it < kBisections && hb - lb > 1; it++) {
             const long long mb = lb + (hb - lb) / 2;
             const double mid = __longlong_as_double(mb);
-            double gm, sm;
-            g_and_slope(c, eta, cp, cw, eps, mid, inv_n, gm, sm);
-            if (sm >= 0.0) { hb = mb; hi = mid; g_hi = gm; }
-            else { lb = mb; lo = mid; g_lo = gm; }
+            if (slope_at(c, eta, cp, cw, eps, mid, inv_n) >= 0.0) { hb = mb; hi = mid; }
+            else { lb = mb; lo = mid; }
         }
         // g is linear between kinks: the better end of the final bracket is the minimum
+        const double g_lo = value_at(c, eta, cp, cw, eps, lo, inv_n), g_hi = value_at(c, eta, cp, cw, eps, hi, inv_n);
         if (g_hi < g_lo) { best_g = g_hi; best_gam = hi; }
         else { best_g = g_lo; best_gam = lo; }
+    } else {
+        best_g = value_at(c, eta, cp, cw, eps, lo, inv_n);  // g rises from gamma = 0
+        best_gam = lo;
     }
     // Every g is at least the empirical cost (1/N) sum Q(eta, x_n): the empirical distribution
     // lies in the ball, and phi >= Q(eta, x) at every gamma.  That bound is exact from integer
