@@ -279,9 +279,11 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
         tma_bulk_load(smem_u32(ring + (size_t)s * C::CHUNK), src + (int64_t)c * C::CHUNK, (uint32_t)(cnt * sizeof(float2)),
                       smem_u32(&full[s]));
     };
+    __shared__ double s_inv_n;  // 1 / N, one FP64 division per CTA (FP64 runs at 1/64 of FP32 here)
     if (tid == 0) {
         for (int s = 0; s < C::STAGES; s++) mbar_init(smem_u32(&full[s]), 1);
         fence_mbar_init();
+        s_inv_n = 1.0 / (double)a.N[k];
     }
     __syncthreads();
     if (tid == 0)
@@ -628,7 +630,7 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
                                         : cw * eta_i * Nk - nu * (double)sx;
                 tot = base + acc64;
             }
-            const double S = tot / Nk;
+            const double S = tot * s_inv_n;
             s_S[(r_local0 + i) * NLpad + lj] = S;
             if (a.S_out) {
                 const size_t o = (((size_t)m * a.K + k) * a.R + ri) * a.NL + lj;

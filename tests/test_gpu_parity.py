@@ -303,6 +303,19 @@ def test_exact_kernel_at_its_largest_support(prec):
     compare_full(w, run(w, P[prec]), O.solve(w), prec)
 
 
+@pytest.mark.parametrize("prec", ["fp32", "fp64"])
+def test_staging_offsets_differ_by_class(prec):
+    """A class staged as x + 2^23 (support at most 2^22) beside one staged as x (support above
+    2^22) in one request: the FP32-arithmetic and FP64 kernels remove each class's own offset."""
+    L_small, L_big = 3000, (1 << 22) + 100
+    rng = np.random.default_rng(31)
+    w = make([np.concatenate([[0, L_small], rng.integers(0, L_small + 1, 2000)]),
+              np.concatenate([[0, 1, L_big], rng.integers(0, L_big + 1, 900)])],
+             [L_small, L_big], [0, 1, 1500, 2999, 3000], np.logspace(-3, 2, 24), [0.0, 300.0], [10.0, 1.0],
+             [1.0, 2.0])
+    compare_full(w, run(w, P[prec]), O.solve(w), prec)
+
+
 @pytest.mark.parametrize("nl", [40, 200])
 def test_fp32_above_the_exact_limit_matches_the_oracle(nl):
     """Supports above 2^22 take the FP32-arithmetic kernel (the exact one needs L <= 2^22)."""
