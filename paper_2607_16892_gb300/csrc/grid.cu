@@ -43,11 +43,13 @@ constexpr int ilog2(int v) { return v <= 1 ? 0 : 1 + ilog2(v / 2); }
 
 // Shape of one instantiation of the grid kernel: precision, warp tile (TR reservations x TL
 // multipliers, TR*TL a power of two <= 32), FP32 chunks between folds of the per-lane partial
-// sums into FP64 (FP64 folds once at the end), and the largest CTA and minimum CTAs per SM it is
-// compiled for (these two bound its registers per thread).
+// sums into FP64 (FP64 folds once at the end), the largest CTA and minimum CTAs per SM it is
+// compiled for (these two bound its registers per thread), the staged chunk and ring depth, the
+// sample loop's unroll, and (exact) the lam columns per row on packed FP32 adds.
 template <Prec P_, int TR_, int TL_, int FLUSH_, int MINB_, int MAXT_ = 512, int CHUNK_ = 2048, int STAGES_ = 3,
-          int UNROLL_ = 2>
+          int UNROLL_ = 2, int FCOLS_ = TL_ / 2>
 struct GridCfg {
+    static constexpr int FCOLS = FCOLS_;
     static constexpr Prec P = P_;
     static constexpr int TR = TR_, TL = TL_, V = TR_ * TL_, LOG2V = ilog2(TR_ * TL_), FLUSH = FLUSH_, MINB = MINB_;
     static constexpr int MAXT = MAXT_;
@@ -63,12 +65,14 @@ struct GridCfg {
 // such warps per SM and the FP32 kernel 2 x 16 tiles.  FP64: 2 x 8 tiles.
 // All stage 4096-sample chunks (32 KB) through a 2-deep ring.  The FP32 variants fold their
 // partial sums every 2 chunks (256 samples per lane); the exact variants fold as often as their
-// support size requires.  The narrow variants unroll the sample loop 8 times.
+// support size requires.  The narrow FP32 variant unrolls the sample loop 8 times, the exact
+// variants 4 times, and the exact variants give half of every row's lam columns (FCOLS) to the
+// packed FP32 adds, the rest to the integer absolute differences.
 using CfgF32 = GridCfg<Prec::F32, 2, 8, 2, 2, 512, 4096, 2, 8>;
 using CfgF32Wide = GridCfg<Prec::F32, 2, 16, 2, 1, 512, 4096, 2, 2>;
 using CfgF64 = GridCfg<Prec::F64, 2, 8, 0, 1, 512, 4096, 2>;
-using CfgExact = GridCfg<Prec::EXACT, 2, 8, 0, 2, 512, 4096, 2, 8>;
-using CfgExactWide = GridCfg<Prec::EXACT, 2, 8, 0, 1, 1024, 4096, 2, 8>;
+using CfgExact = GridCfg<Prec::EXACT, 2, 8, 0, 2, 512, 4096, 2, 4>;
+using CfgExactWide = GridCfg<Prec::EXACT, 2, 8, 0, 1, 1024, 4096, 2, 4>;
 constexpr int kWarpsTarget = 16;  // warps per CTA the r groups fill up to
 
 // ---------------------------------------------------------------- PTX helpers
@@ -441,14 +445,13 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
         // packed FP32 add forms y = x' + (1 - t - 2^23) = x - c for two cells and one adds |y| into
         // the running sum (the absolute value rides on the add's operand); for the other half one
         // integer absolute-difference-and-add (__sad) works on the staged float's bit pattern,
-        // 0x4B000000 + x.  The two kinds alternate in the instruction stream.  Every value is an
-        // integer below 2^24, so both are exact.  Sums are folded into int64 through the warp
-        // transposition before an FP32 sum could pass 2^24.  The count #{x >= t} comes from the
-        // class's cumulative counts; the epilogue puts every sample on its branch of phi with these
-        // integer sums (branch_sum) in FP64.
-        constexpr int TLF = TL / 2;  // lam columns per r row on the packed FP32 adds (in pairs)
+        // 0x4B000000 + x.  Every value is an integer below 2^24, so both are exact.  Sums are
+        // folded into int64 through the warp transposition before an FP32 sum could pass 2^24.  The
+        // count #{x >= t} comes from the class's cumulative counts; the epilogue puts every sample
+        // on its branch of phi with these integer sums (branch_sum) in FP64.
+        constexpr int TLF = C::FCOLS;  // lam columns per r row on the packed FP32 adds (in pairs)
         constexpr int TLI = TL - TLF;  // lam columns per r row on the integer path
-        static_assert(TLF % 2 == 0 && TLI == TLF, "pairs of packed columns alternate with pairs of integer ones");
+        static_assert(TLF % 2 == 0 && TLF >= 2 && TLI >= 1, "packed columns come in pairs");
         u64 ntf[TR][TLF / 2], accf[TR][TLF / 2];  // ntf: 1 - t - 2^23 for a pair of cells
         int cci[TR][TLI];                          // 0x4B000000 + t - 1 per cell
         unsigned acci[TR][TLI];
@@ -505,25 +508,19 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
             }
             acc_r += (long long)transpose_reduce<unsigned, V>(vs, lane);
         };
-        // one load: two samples' (x', x') pairs into every cell's sum; a pair of packed columns
-        // alternates with a pair of integer columns, add for add
+        // one load: two samples' (x', x') pairs into every cell's sum (the compiler interleaves the
+        // two pipes' instructions)
         auto step = [&](const float4 v) {
             const u64 xa = pk(v.x, v.y), xb = pk(v.z, v.w);
             const int ba = __float_as_int(v.x), bb = __float_as_int(v.z);  // 0x4B000000 + x
 #pragma unroll
-            for (int i = 0; i < TR; i++)
+            for (int i = 0; i < TR; i++) {
 #pragma unroll
-                for (int p = 0; p < TLF / 2; p++) {
-                    const int j0 = 2 * p, j1 = 2 * p + 1;
-                    const u64 ya = fadd2(xa, ntf[i][p]);
-                    acci[i][j0] = __sad(ba, cci[i][j0], acci[i][j0]);
-                    const u64 yb = fadd2(xb, ntf[i][p]);
-                    acci[i][j1] = __sad(ba, cci[i][j1], acci[i][j1]);
-                    const u64 sy = fadd2(abs2(ya), abs2(yb));
-                    acci[i][j0] = __sad(bb, cci[i][j0], acci[i][j0]);
-                    accf[i][p] = fadd2(accf[i][p], sy);
-                    acci[i][j1] = __sad(bb, cci[i][j1], acci[i][j1]);
-                }
+                for (int p = 0; p < TLF / 2; p++)
+                    accf[i][p] = fadd2(accf[i][p], fadd2(abs2(fadd2(xa, ntf[i][p])), abs2(fadd2(xb, ntf[i][p]))));
+#pragma unroll
+                for (int jj = 0; jj < TLI; jj++) acci[i][jj] = __sad(bb, cci[i][jj], __sad(ba, cci[i][jj], acci[i][jj]));
+            }
         };
         auto run = [&](const float4* q, int t0, int t1, bool clamp) {
             if (clamp) {
