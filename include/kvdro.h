@@ -58,10 +58,11 @@ typedef enum {
                             results rounded to FP32 (the exact kernel is also the fastest);
                             otherwise per-term arithmetic in FP32 with sums folded into FP64 */
     KVDRO_FP64 = 1,      /* per-term arithmetic and sums in FP64 */
-    KVDRO_EXACT = 2,     /* per term, FP32 integer arithmetic on exact integer thresholds
-                            (|x + 1 - t| summed exactly); exact integer counts and sums combined
-                            once per cell in FP64, so results carry FP64 rounding only.  Needs
-                            every L_max <= 2^22. */
+    KVDRO_EXACT = 2,     /* per term, exact integer arithmetic on exact integer thresholds
+                            (|x + 1 - t| summed exactly, half of the cells in packed FP32 adds,
+                            half in integer absolute differences); exact integer counts and
+                            sums combined once per cell in FP64, so results carry FP64 rounding
+                            only.  Needs every L_max <= 2^22. */
     KVDRO_ENVELOPE = 3   /* not per term: each cell's sample sum from the sorted samples'
                             cumulative counts and sums at its exact threshold, O(1) per cell,
                             FP64 outputs with FP64 rounding only */
