@@ -55,10 +55,11 @@ struct GridCfg {
     static constexpr int MAXT = MAXT_;
     static constexpr int CHUNK = CHUNK_;    // samples per staged chunk (float2 each)
     static constexpr int STAGES = STAGES_;  // ring depth
-    static constexpr int UNROLL = UNROLL_;  // unroll of the FP32 sample loop
+    static constexpr int UNROLL = UNROLL_;  // unroll of the sample loop
     static_assert(CHUNK_ % 128 == 0 && CHUNK_ * 8 * STAGES_ <= 160 * 1024, "chunk ring must fit shared memory");
     static_assert((V & (V - 1)) == 0 && V >= 2 && V <= 32, "tile must hold a power of two <= 32 cells");
     static_assert(P_ == Prec::F64 || TL_ % 2 == 0, "the FP32 and exact tiles pack lam values in pairs");
+    static_assert(FLUSH >= 0 && UNROLL >= 1 && FCOLS >= 0 && FCOLS <= TL, "shape parameters out of range");
 };
 // 2 r x 8 lam tiles, up to 16 warps per CTA and (FP32, exact) two CTAs per SM (64 registers)
 // for up to 128 lam values; for 129..256 lam values the exact kernel runs one CTA of up to 32
@@ -84,14 +85,6 @@ __device__ __forceinline__ u64 pk(float lo, float hi) {
 }
 __device__ __forceinline__ void upk(u64 r, float& lo, float& hi) {
     asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(r));
-}
-__device__ __forceinline__ u64 pki(unsigned lo, unsigned hi) {
-    u64 r;
-    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "r"(lo), "r"(hi));
-    return r;
-}
-__device__ __forceinline__ void upki(u64 r, unsigned& lo, unsigned& hi) {
-    asm("mov.b64 {%0, %1}, %2;" : "=r"(lo), "=r"(hi) : "l"(r));
 }
 __device__ __forceinline__ u64 ffma2(u64 a, u64 b, u64 c) {
     u64 r;
