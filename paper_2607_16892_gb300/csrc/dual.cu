@@ -47,17 +47,18 @@ __device__ __forceinline__ void split_at(const ClassView& c, double eta, double 
     tail(c, first_active(mu + nu, excess_offset(cp, cw, mu, (double)c.L, eta), c.L), cnt, sum);
 }
 
-// Right derivative of g at gamma: the active set just above gamma is the one at gamma up to
-// samples whose excess is exactly zero, which change the value by nothing and the slope only at
-// a kink.  Only its sign steers the bisection.
-__device__ __forceinline__ double slope_at(const ClassView& c, double eta, double cp, double cw, double eps,
-                                           double gam, double inv_n) {
+// Sign of the right derivative of g at gamma, eps - (nu' sum_{x < t} x + mu' sum_{x >= t} (L - x)) / N
+// with nu' = [gamma < c_w], mu' = [gamma < c_p]: the active set just above gamma is the one at
+// gamma up to samples whose excess is exactly zero, which change the value by nothing and the
+// slope only at a kink.  Tested as eps N >= the integer sum (eps_n = eps N rounded once), the
+// sign is all the bisection needs.
+__device__ __forceinline__ bool slope_nonneg(const ClassView& c, double eta, double cp, double cw, double eps_n,
+                                             double gam) {
     double mu, nu;
     int64_t cnt, sum;
     split_at(c, eta, cp, cw, gam, mu, nu, cnt, sum);
-    const double dmu = gam < cp ? 1.0 : 0.0, dnu = gam < cw ? 1.0 : 0.0;
-    const int64_t below = c.sumx - sum, dist = (int64_t)c.L * cnt - sum;  // sum x below t, sum (L - x) from t on
-    return eps - (dnu * (double)below + dmu * (double)dist) * inv_n;
+    const int64_t drop = (gam < cw ? c.sumx - sum : 0) + (gam < cp ? (int64_t)c.L * cnt - sum : 0);
+    return eps_n >= (double)drop;
 }
 
 // g(gamma) = gamma eps + S(eta, gamma), every sample on its own branch of phi.
@@ -90,14 +91,15 @@ __global__ void __launch_bounds__(kDualThreads) k_dual(const DualArgs a) {
     const double cp = a.cp[m], cw = a.cw[m], eps = a.eps[e];
     const double eta = (double)a.r[ri] - (double)a.L_in[k];
     const double inv_n = 1.0 / (double)c.N;
+    const double eps_n = eps * (double)c.N;
     double lo = 0.0, hi = fmax(cp, cw);
     double best_g, best_gam;
-    if (slope_at(c, eta, cp, cw, eps, lo, inv_n) < 0.0 && hi > 0.0) {
+    if (!slope_nonneg(c, eta, cp, cw, eps_n, lo) && hi > 0.0) {
         long long lb = __double_as_longlong(lo), hb = __double_as_longlong(hi);  // 0 <= lb < hb < 2^63
         for (int it = 0; it < kBisections && hb - lb > 1; it++) {
             const long long mb = lb + (hb - lb) / 2;
             const double mid = __longlong_as_double(mb);
-            if (slope_at(c, eta, cp, cw, eps, mid, inv_n) >= 0.0) { hb = mb; hi = mid; }
+            if (slope_nonneg(c, eta, cp, cw, eps_n, mid)) { hb = mb; hi = mid; }
             else { lb = mb; lo = mid; }
         }
         // g is linear between kinks: the better end of the final bracket is the minimum

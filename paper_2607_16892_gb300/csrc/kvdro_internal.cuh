@@ -146,9 +146,13 @@ cudaError_t launch_dual(const DualArgs& a, cudaStream_t s);
 // c_p (L - eta) - (mu L + c_w eta): L - eta is an exact integer and every product is rounded once,
 // so a large c_p never swallows a small mu or c_w (the first form cancels to 0 at eta = L when
 // mu and c_w are far below c_p, though d is then -(mu + c_w) L).  At the saturated multiplier
-// mu = c_p the L terms vanish exactly and d = -(c_p + c_w) eta.
+// mu = c_p the L terms vanish exactly and d = -(c_p + c_w) eta.  Every rounding is spelled out
+// (no contraction left to the compiler), so each call site gets the same d bit for bit: a
+// kernel that classifies samples twice at one multiplier (the dual's slope and value) must see
+// the same threshold both times.
 __device__ __forceinline__ double excess_offset(double cp, double cw, double mu, double L, double eta) {
-    return mu == cp ? -(cp * eta + cw * eta) : cp * (L - eta) - (mu * L + cw * eta);
+    const double cw_eta = __dmul_rn(cw, eta);
+    return mu == cp ? -__fma_rn(cp, eta, cw_eta) : __dsub_rn(__dmul_rn(cp, L - eta), __fma_rn(mu, L, cw_eta));
 }
 
 // sum_n phi(x_n) with every sample on its own branch: V = c_w eta - nu x for the n - cnt samples
