@@ -12,15 +12,23 @@
 // so phi = max(U, V) = V + max(W, 0) with W = U - V = kappa x + d,
 //   kappa = mu + nu,   d = (c_p - mu) L - (c_p + c_w) eta.
 // Summing over the class: sum_n phi_n = N c_w eta - nu sum_n x_n + sum_n max(kappa x_n + d, 0).
-// The first two terms are exact from the class's integer sample sum; the kernel evaluates the
-// last one term by term: one fused multiply-add, one max and one add per (sample, cell).
+// Three forms of that sum:
+//  - FP32 and FP64 per term: the excess max(kappa x + d, 0) term by term (one fused multiply-add,
+//    one max, one add per sample and cell) on the base V, or max(-(kappa x + d), 0) on the base
+//    U when nu > mu, whichever cancels less (use_u_split).
+//  - EXACT (also FP32 requests whose supports are all <= 2^22): each cell's integer threshold t
+//    (x >= t exactly when kappa x + d > 0), then per term the exact sum of |x + 1 - t|, half of a
+//    warp's cells on packed FP32 adds and half on integer absolute differences, so the FMA and ALU
+//    pipes work side by side; the epilogue puts every sample on its own branch (branch_sum).
+//  - ENVELOPE (k_envelope): the same branch sums from the cumulative counts and sums, O(1) per
+//    cell, not per term.
 //
 // Work decomposition.  A CTA owns one (regime m, class k) and a block of RG*TR consecutive r
 // values for the whole lam grid.  Each warp owns a TR x TL tile of (r, lam) cells; its 32 lanes
 // split the class's samples, which stream through a ring of shared-memory chunks filled by TMA
-// bulk copies (cp.async.bulk + mbarrier).  The FP32 path packs two cells per f32x2 instruction.
-// Every chunk, each lane's FP32 partial sums are transposed and reduced across the warp
-// (fixed shuffle order) so that each lane then owns one cell, folded into an FP64 accumulator.
+// bulk copies (cp.async.bulk + mbarrier).  Packed f32x2 instructions serve two cells at once.
+// Periodically each lane's partial sums are transposed and reduced across the warp (fixed
+// shuffle order) so that each lane then owns one cell, folded into an FP64 or int64 accumulator.
 // The epilogue forms S = (1/N) sum phi, then for every eps the minimum over lam (lowest index),
 // and feeds the argmin over r through a 64-bit atomicMin on (cost, r index) keys.
 #include <float.h>
