@@ -127,7 +127,9 @@ int kvdro_eval_grid(kvdro_ctx* ctx, int precision, int32_t R, const int32_t* r, 
  * and piecewise linear in gamma with its minimiser in [0, max(c_p, c_w)]; the library bisects on
  * its right derivative over the ordered bit patterns of the nonnegative doubles (at most 63
  * steps, down to two adjacent doubles at any scale) with every evaluation O(1) from the sorted
- * samples' cumulative counts and sums, so results carry FP64 rounding only.
+ * samples' cumulative counts and sums, so results carry FP64 rounding only.  The result is
+ * never below the empirical cost (1/N) sum_n Q(eta, x_n), computed exactly from integer sums:
+ * that bound holds at every gamma (App. A) and is the value itself at eps = 0.
  * Arguments as kvdro_eval_grid; outputs (each may be NULL; host or device):
  *   cost       double [M][E][K][R]   the exact dual value
  *   gamma      double [M][E][K][R]   a minimising gamma
