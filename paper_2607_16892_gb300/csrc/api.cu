@@ -438,7 +438,11 @@ int kvdro_eval_grid(kvdro_ctx* ctx, int precision, int32_t R, const int32_t* r, 
                  : precision == KVDRO_EXACT ? Prec::EXACT : Prec::ENVELOPE;
     const int32_t maxNL = P == Prec::F64 ? kMaxNLf64 : kMaxNLf32;
     bool exact_ok = true;  // every class's support fits the exact kernel's integer sums
-    for (int32_t k = 0; k < ctx->K; k++) exact_ok = exact_ok && ctx->L[k] <= kvdro::kExactMaxL;
+    int32_t max_L = 0;
+    for (int32_t k = 0; k < ctx->K; k++) {
+        exact_ok = exact_ok && ctx->L[k] <= kvdro::kExactMaxL;
+        max_L = std::max(max_L, ctx->L[k]);
+    }
     if (P == Prec::EXACT && !exact_ok)
         return fail(ctx, KVDRO_EINVAL, "KVDRO_EXACT needs L_max <= 2^22 for every class");
     // FP32 results come from the exact kernel (rounded to FP32) whenever it applies: it is exact
@@ -465,7 +469,7 @@ int kvdro_eval_grid(kvdro_ctx* ctx, int precision, int32_t R, const int32_t* r, 
     ctx->last_stream = s;
 
     // Launch shape: lam tiles x r groups of warps per CTA.
-    const kvdro::GridShape shape = kvdro::grid_shape(KP, R, NL, E);
+    const kvdro::GridShape shape = kvdro::grid_shape(KP, R, NL, E, max_L);
 
     // Grid parameters in one upload.
     const size_t gbytes = align_up((size_t)R * 4, 8) + 8 * ((size_t)NL + E + 2 * (size_t)M);

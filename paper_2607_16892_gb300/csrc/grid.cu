@@ -82,6 +82,11 @@ using CfgF32Wide = GridCfg<Prec::F32, 2, 16, 2, 1, 512, 4096, 2, 2>;
 using CfgF64 = GridCfg<Prec::F64, 2, 8, 0, 1, 512, 4096, 2>;
 using CfgExact = GridCfg<Prec::EXACT, 2, 8, 0, 2, 512, 4096, 2, 4>;
 using CfgExactWide = GridCfg<Prec::EXACT, 2, 8, 0, 1, 1024, 4096, 2, 4>;
+// Above a support of 2^19 the packed FP32 sums (exact only up to 2^24) would fold every few loads;
+// there every column takes the integer absolute differences, whose sums fold far less often.
+using CfgExactInt = GridCfg<Prec::EXACT, 2, 8, 0, 2, 512, 4096, 2, 8, 0>;
+using CfgExactIntWide = GridCfg<Prec::EXACT, 2, 8, 0, 1, 1024, 4096, 2, 8, 0>;
+constexpr int32_t kExactIntAboveL = 1 << 19;
 constexpr int kWarpsTarget = 16;  // warps per CTA the r groups fill up to
 
 // ---------------------------------------------------------------- PTX helpers
@@ -452,8 +457,9 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
         // on its branch of phi with these integer sums (branch_sum) in FP64.
         constexpr int TLF = C::FCOLS;  // lam columns per r row on the packed FP32 adds (in pairs)
         constexpr int TLI = TL - TLF;  // lam columns per r row on the integer path
-        static_assert(TLF % 2 == 0 && TLF >= 2 && TLI >= 1, "packed columns come in pairs");
-        u64 ntf[TR][TLF / 2], accf[TR][TLF / 2];  // ntf: 1 - t - 2^23 for a pair of cells
+        static_assert(TLF % 2 == 0 && TLI >= 1, "packed columns come in pairs");
+        constexpr int NPF = TLF > 0 ? TLF / 2 : 1;  // array extent (unused when TLF = 0)
+        u64 ntf[TR][NPF], accf[TR][NPF];           // ntf: 1 - t - 2^23 for a pair of cells
         int cci[TR][TLI];                          // 0x4B000000 + t - 1 per cell
         unsigned acci[TR][TLI];
         // Each lane works out the threshold of the cell it owns after the final transposition
@@ -483,11 +489,13 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
                 acci[i][jj] = 0u;
             }
         }
-        // Fold after `fe` loads of two samples: a lane's sums are then at most 2 fe (L + 1) <= 2^24,
-        // exact in FP32, and the transposition's 32-lane sums stay below 2^29; fe is a power of two,
-        // the same for every thread of the CTA.
+        // Fold after `fe` loads of two samples, when a lane's sums are at most 2 fe (L + 1): with
+        // packed columns that is at most 2^24 (exact in FP32; the transposition's 32-lane sums stay
+        // below 2^29); with none, only the integer limit applies (32 lanes' sums below 2^32).  fe
+        // is a power of two, the same for every thread of the CTA.
+        const int64_t fold_lim = TLF > 0 ? (1ll << 24) : (1ll << 32) / 32 - 1;
         int fe = 1;
-        while (fe < (1 << 20) && 2ll * (2 * fe) * ((int64_t)a.L[k] + 1) <= (1ll << 24)) fe <<= 1;
+        while (fe < (1 << 20) && 2ll * (2 * fe) * ((int64_t)a.L[k] + 1) <= fold_lim) fe <<= 1;
         long long acc_r = 0;
         auto fold = [&]() {
             unsigned vs[V];
@@ -728,7 +736,7 @@ GridShape shape_for(int variant, int32_t R, int32_t NL, int32_t E) {
     return sh;
 }
 
-GridShape grid_shape(Prec p, int32_t R, int32_t NL, int32_t E) {
+GridShape grid_shape(Prec p, int32_t R, int32_t NL, int32_t E, int32_t max_L) {
     if (p == Prec::ENVELOPE) {
         GridShape sh;
         sh.variant = 4;
@@ -740,8 +748,12 @@ GridShape grid_shape(Prec p, int32_t R, int32_t NL, int32_t E) {
         return sh;
     }
     if (p == Prec::F64) return shape_for<CfgF64>(2, R, NL, E);
-    if (p == Prec::EXACT)
-        return NL <= kWarpsTarget * CfgExact::TL ? shape_for<CfgExact>(3, R, NL, E) : shape_for<CfgExactWide>(5, R, NL, E);
+    if (p == Prec::EXACT) {
+        const bool narrow = NL <= kWarpsTarget * CfgExact::TL;
+        if (max_L > kExactIntAboveL)
+            return narrow ? shape_for<CfgExactInt>(6, R, NL, E) : shape_for<CfgExactIntWide>(7, R, NL, E);
+        return narrow ? shape_for<CfgExact>(3, R, NL, E) : shape_for<CfgExactWide>(5, R, NL, E);
+    }
     if (NL <= kWarpsTarget * CfgF32::TL) return shape_for<CfgF32>(0, R, NL, E);
     return shape_for<CfgF32Wide>(1, R, NL, E);
 }
@@ -752,8 +764,10 @@ cudaError_t grid_prepare(Prec p) {
     if (p == Prec::F64) return cudaFuncSetAttribute(k_grid<CfgF64>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
     if (p == Prec::EXACT) {
         cudaError_t e = cudaFuncSetAttribute(k_grid<CfgExact>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
-        if (e != cudaSuccess) return e;
-        return cudaFuncSetAttribute(k_grid<CfgExactWide>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
+        if (e == cudaSuccess) e = cudaFuncSetAttribute(k_grid<CfgExactWide>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
+        if (e == cudaSuccess) e = cudaFuncSetAttribute(k_grid<CfgExactInt>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
+        if (e == cudaSuccess) e = cudaFuncSetAttribute(k_grid<CfgExactIntWide>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
+        return e;
     }
     if (p == Prec::ENVELOPE)
         return cudaFuncSetAttribute(k_envelope, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -781,7 +795,9 @@ cudaError_t launch_grid(Prec p, const GridShape& sh, GridArgs a, cudaStream_t s)
     if (p == Prec::ENVELOPE) k_envelope<<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
     else if (p == Prec::F64) k_grid<CfgF64><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
     else if (p == Prec::EXACT && sh.variant == 3) k_grid<CfgExact><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
-    else if (p == Prec::EXACT) k_grid<CfgExactWide><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
+    else if (p == Prec::EXACT && sh.variant == 5) k_grid<CfgExactWide><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
+    else if (p == Prec::EXACT && sh.variant == 6) k_grid<CfgExactInt><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
+    else if (p == Prec::EXACT) k_grid<CfgExactIntWide><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
     else if (sh.variant == 0) k_grid<CfgF32><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
     else k_grid<CfgF32Wide><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
     return cudaGetLastError();

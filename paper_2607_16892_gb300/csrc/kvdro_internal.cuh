@@ -111,7 +111,7 @@ struct GridShape {
     int r_blocks;      // CTAs per (m, k)
     size_t smem;
 };
-GridShape grid_shape(Prec p, int32_t R, int32_t NL, int32_t E);
+GridShape grid_shape(Prec p, int32_t R, int32_t NL, int32_t E, int32_t max_L);  // max_L: largest support
 cudaError_t grid_prepare(Prec p);             // per-device attribute setup of every variant of p
 // Launches over regimes [a.m0, a.m0 + a.m_count); fills a.LT, a.RG, a.r_blocks from `sh`.
 cudaError_t launch_grid(Prec p, const GridShape& sh, GridArgs a, cudaStream_t s);

@@ -261,9 +261,13 @@ extern "C" int kvdro_eval_grid_noalloc(int32_t K, const int64_t* offsets, const 
     // ---- the grid kernel (the exact one, FP32 outputs, whenever every support is at most 2^22;
     // else the FP32-arithmetic one) and the argmin finalisation
     bool exact_ok = true;
-    for (int32_t k = 0; k < K; k++) exact_ok = exact_ok && L_max[k] <= kvdro::kExactMaxL;
+    int32_t max_L = 0;
+    for (int32_t k = 0; k < K; k++) {
+        exact_ok = exact_ok && L_max[k] <= kvdro::kExactMaxL;
+        max_L = L_max[k] > max_L ? L_max[k] : max_L;
+    }
     const kvdro::Prec kp = exact_ok ? kvdro::Prec::EXACT : kvdro::Prec::F32;
-    const kvdro::GridShape shape = kvdro::grid_shape(kp, R, NL, E);
+    const kvdro::GridShape shape = kvdro::grid_shape(kp, R, NL, E, max_L);
     kvdro::GridArgs a;
     a.pairs = sa.pairs;
     a.pair_off = sa.pair_off;

@@ -303,6 +303,18 @@ def test_exact_kernel_at_its_largest_support(prec):
     compare_full(w, run(w, P[prec]), O.solve(w), prec)
 
 
+@pytest.mark.parametrize("L,nl", [(1 << 19, 40), ((1 << 19) + 1, 40), ((1 << 20) + 3, 200)])
+def test_exact_variants_either_side_of_the_integer_split(L, nl):
+    """Supports up to 2^19 run half of every row's columns on packed FP32 adds; above, every
+    column on integer absolute differences (narrow tiles, and wide ones for 200 lam values).
+    Both forms are exact."""
+    rng = np.random.default_rng(41)
+    w = make([np.concatenate([[0, L], rng.integers(0, L + 1, 3000)]), rng.integers(L - 9000, L + 1, 500)], L,
+             [0, 1, L // 3, L - 1, L], np.logspace(-3, 2, nl), [0.0, 700.0], [10.0, 0.5], [1.0, 3.0])
+    compare_full(w, run(w, kvdro.KVDRO_EXACT), O.solve(w), "exact")
+    compare_full(w, run(w, kvdro.KVDRO_FP32), O.solve(w), "fp32")
+
+
 @pytest.mark.parametrize("prec", ["fp32", "fp64"])
 def test_staging_offsets_differ_by_class(prec):
     """A class staged as x + 2^23 (support at most 2^22) beside one staged as x (support above
