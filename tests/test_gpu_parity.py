@@ -315,6 +315,17 @@ def test_exact_variants_either_side_of_the_integer_split(L, nl):
     compare_full(w, run(w, kvdro.KVDRO_FP32), O.solve(w), "fp32")
 
 
+def test_integer_variant_with_input_lengths_and_ragged_classes():
+    """The all-integer variant (support above 2^19) with per-class input lengths, a class of 1 and
+    one of 67 samples (padding in its only load), and a support point at each end."""
+    L = (1 << 20) + 17
+    rng = np.random.default_rng(43)
+    w = make([np.concatenate([[0, L], rng.integers(0, L + 1, 2047)]), [L // 2], rng.integers(0, L + 1, 67)], L,
+             [40, 41, 5000, L // 2, L], np.logspace(-2, 1.5, 29), [0.0, 3.0, 9000.0], [4.0, 1.0, 0.25],
+             [1.0, 2.0, 1.0], L_in=[40, 0, 7])
+    compare_full(w, run(w, kvdro.KVDRO_EXACT), O.solve(w), "exact")
+
+
 @pytest.mark.parametrize("prec", ["fp32", "fp64"])
 def test_staging_offsets_differ_by_class(prec):
     """A class staged as x + 2^23 (support at most 2^22) beside one staged as x (support above
