@@ -1,14 +1,15 @@
 #!/usr/bin/env python3
 """Throughput of the Wasserstein-DRO reservation-cost path on one GB300 (or N replicas).
 
-One step is one pass of the whole path over the 8-class lognormal workload
-(8 classes x 100,000 samples, 4096 reservations x 128 multipliers x 8 radii,
-c_p/c_w = 10): load + range check + segmented sort of the samples, 5 quantiles,
-the FP32 grid evaluation with its eps epilogue, and the argmin over r.  The
-metric counts one cost term per (class, r, lam, sample) per regime; eps does not
-multiply per-sample work and is not counted.
+One step is one pass of the whole path over the regime-sweep workload, the largest of the
+five workload configurations (8 classes x 200,000 samples; 2048 reservations x 64
+multipliers x 16 radii x 1024 cost regimes c_p/c_w log-spaced over [1, 1000]; 2.15e14 cost
+terms): load + range check + segmented sort of the samples, the 1024 critical-fractile
+quantiles, the FP32 grid evaluation with its eps epilogue, and the argmin over r.  The
+metric counts one cost term per (regime, class, r, lam, sample); eps does not multiply
+per-sample work and is not counted.
 
-  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference] [--workload NAME]
 
 Under torchrun each rank evaluates its own replica of the workload (independent
 problems, no collective on the data path); the JSON line reports the sum of all
@@ -22,6 +23,7 @@ import argparse
 import hashlib
 import json
 import os
+import platform
 import re
 import statistics
 import subprocess
@@ -34,10 +36,11 @@ import numpy as np
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
-from synth import lognormal_workload_k8_n1e5, slice_workload  # noqa: E402
+from synth import WORKLOADS, slice_workload  # noqa: E402
 
 METRIC = "DRO cost terms/sec (class×r×λ×sample) on 1 GB300; % of FP32/HBM roofline"
 UNIT = "terms/s"
+DEFAULT_WORKLOAD = "regimes_k8_n2e5"
 SM_MAX_MHZ_RECIPE = 2070.0
 # Bound of the exact kernel's per-term work.  A term costs one instruction-lane on one of two
 # pipes: packed f32x2 adds on the FMA pipe (128 FP32 lanes/clk/SM, two lane-operations per term:
@@ -49,8 +52,17 @@ SM_MAX_MHZ_RECIPE = 2070.0
 FMA_TERMS_PER_CLK_PER_SM = 128.0 / 2.0
 ALU_TERMS_PER_CLK_PER_SM = 64.0
 TERMS_PER_CLK_PER_SM = FMA_TERMS_PER_CLK_PER_SM + ALU_TERMS_PER_CLK_PER_SM
+# The per-term bound of the three-candidate supremum as written: two FMAs, two maxima and one add
+# per term, 5 FP32 lane-operations on 128 FP32 lanes per clock per SM.
+PAPER_FORM_LANE_OPS_PER_TERM = 5.0
+# What the exact kernel evaluates per term: once a cell's exact integer threshold t is known
+# (x >= t exactly when the excess kappa x + d is positive), the excess sum is
+# kappa sum_{x >= t} x + d #{x >= t}, and the kernel streams sum_n |x_n - (t - 1)| to get it.
+# That sum also has an O(1) closed form from the cumulative counts and sums the same context holds
+# (the envelope mode returns the same S that way).
+PER_TERM_OP = "|x - c| summed exactly per (cell, sample), c = t - 1 the cell's integer threshold; not the 3-candidate phi"
 GRID_SOURCE = os.path.join(ROOT, "paper_2607_16892_gb300", "csrc", "grid.cu")
-PROFILE = os.path.join(ROOT, "profiles", "k_grid_exact_lognormal_k8_n1e5.md")
+PROFILE = os.path.join(ROOT, "profiles", "k_grid_exact_regimes_k8_n2e5.md")
 LAUNCHES_PER_STEP = 7  # histogram, scan totals, scan, expand, quantile gather, grid, argmin finalise
 # FP64 pipe bound of the native FP64 mode: per term one DFMA (2.0 per clk per SM) plus one DADD and
 # one max.f64 (1.7 per clk per SM each), measured on this GB300; nominal 1.25 TFLOP/s FP64.
@@ -60,22 +72,25 @@ FP64_TERMS_PER_CLK_PER_SM = 1.0 / (1.0 / 2.0 + 2.0 / 1.7)
 def parse_args():
     p = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     p.add_argument("--gpus", type=int, default=1)
-    p.add_argument("--steps", type=int, default=100)
-    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--steps", type=int, default=5)
+    p.add_argument("--warmup", type=int, default=3)
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    p.add_argument("--e2e-steps", type=int, default=30)
+    p.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(WORKLOADS),
+                   help="workload configuration of a step (default: the largest, the regime sweep)")
+    p.add_argument("--e2e-steps", type=int, default=2)
     p.add_argument("--cpu-seconds", type=float, default=10.0, help="target wall time of the CPU-baseline sample")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--drift-iterations", type=int, default=3)
     p.add_argument("--case", default="",
-                   help="WORKLOAD:MODE, MODE in fp32|fp64|exact|envelope|dual|sort: time one kernel path "
-                        "(--warmup untimed, --steps timed runs) and print one line per run")
+                   help="WORKLOAD:MODE[:key=val,...], MODE in fp32|fp64|exact|envelope|dual|sort: time one kernel "
+                        "path (--warmup untimed, --steps timed runs) and print one line per run.  Keys: L (support "
+                        "declared for every class, e.g. 4194305 so FP32 requests take the FP32-arithmetic kernel), "
+                        "nl (lam count, log-spaced over the workload's lam range), m (first m regimes), "
+                        "rstride (every rstride-th r)")
     p.add_argument("--suite", action="store_true",
                    help="time every workload in each precision (one JSON line per case) instead of the contract line")
     p.add_argument("--cpu-suite", action="store_true",
                    help="time the CPU oracle (the reported baseline) on every workload, one line each")
-    p.add_argument("--bcd", action="store_true",
-                   help="time the block-coordinate descent (Alg. 1) on the scalability instances, one line each")
     return p.parse_args()
 
 
@@ -84,6 +99,7 @@ def dist_env():
 
 
 def workload_config(w, world):
+    ratio = w.cp / w.cw
     return {
         "workload": w.name,
         "classes": int(w.K),
@@ -92,14 +108,37 @@ def workload_config(w, world):
         "lam_points": int(len(w.lam)),
         "eps_points": int(len(w.eps)),
         "regimes": int(len(w.cp)),
-        "cost_ratio": float(w.cp[0] / w.cw[0]),
+        "cost_ratio": float(ratio[0]) if len(ratio) == 1 else f"{len(ratio)} log-spaced in "
+                                                              f"[{ratio.min():g}, {ratio.max():g}]",
         "support_L": int(w.L[0]),
         "fractiles": int(len(w.fractiles)),
         "terms_per_step_per_gpu": int(w.terms()),
         "step": "load+range check+segmented sort, quantiles, FP32 grid eval + eps epilogue + argmin over r",
+        "outputs": "cost and lam index per (regime, eps, class, r); r index, min cost and F-hat per "
+                   "(regime, eps, class); quantiles per (class, fractile)",
         "l2": "flushed between timed steps (256 MiB device write outside the timed events)",
         "parallelism": "single GPU" if world == 1 else f"{world} independent replicas (no data-path collective)",
     }
+
+
+def cpu_model() -> str:
+    """The host CPU's model name (lscpu, else /proc/cpuinfo, else the architecture)."""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        fields = {ln.split(":", 1)[0].strip(): ln.split(":", 1)[1].strip() for ln in out.splitlines() if ":" in ln}
+        name = fields.get("Model name", "")
+        if name and name != "-":
+            vendor = fields.get("Vendor ID", "")
+            return f"{vendor} {name}".strip() if vendor and vendor not in name else name
+    except (OSError, subprocess.SubprocessError):
+        pass
+    try:
+        for line in open("/proc/cpuinfo"):
+            if line.lower().startswith(("model name", "cpu part")):
+                return line.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    return platform.machine()
 
 
 # ------------------------------------------------------------------ clocks
@@ -174,47 +213,54 @@ def weak_scaling_value(terms_per_rank_step: int, steps: int, world: int, slowest
     return terms_per_rank_step * steps * world / slowest_s
 
 
-def profile_traffic():
-    """DRAM bytes per grid-kernel launch from the committed ncu summary, if it was taken
-    on the current kernel source (else None)."""
+def profile_figures():
+    """DRAM bytes per grid-kernel launch and warp instructions per term-lane from the committed
+    ncu summary, if it was taken on the current kernel source (else None for both)."""
     try:
         text = open(PROFILE).read()
         src_hash = hashlib.sha256(open(GRID_SOURCE, "rb").read()).hexdigest()
     except OSError:
-        return None
+        return None, None
     m_hash = re.search(r"grid_cu_sha256:\s*([0-9a-f]{64})", text)
+    if not m_hash or m_hash.group(1) != src_hash:
+        return None, None
     m_traf = re.search(r"traffic_bytes_per_launch:\s*([0-9.eE+]+)", text)
-    if not m_hash or not m_traf or m_hash.group(1) != src_hash:
-        return None
-    return float(m_traf.group(1))
+    m_inst = re.search(r"inst_per_term:\s*([0-9.eE+]+)", text)
+    return (float(m_traf.group(1)) if m_traf else None), (float(m_inst.group(1)) if m_inst else None)
+
+
+def oracle_rows(w, rows: int):
+    """Cells of `rows` (regime, r) rows strided over the workload's M x R rows, each with every
+    class and every lam value: the bounded sample the CPU oracle is timed on."""
+    M, K, R, NL = len(w.cp), w.K, len(w.r), len(w.lam)
+    pick = np.linspace(0, M * R - 1, rows).round().astype(np.int64)
+    m, ri = np.divmod(pick, R)
+    mm = np.repeat(m, K * NL)
+    kk = np.tile(np.repeat(np.arange(K), NL), rows)
+    rr = np.repeat(ri, K * NL)
+    ll = np.tile(np.arange(NL), rows * K)
+    return (mm.astype(np.int32), kk, rr, ll), int(rows * NL * int(w.N.sum()))
 
 
 def cpu_baseline(w, seconds: float):
-    """The CPU oracle (direct per-term FP64 evaluation, all host cores) on a bounded,
-    strided slice of the workload's (class, r) rows with the full lam grid and all samples."""
+    """The CPU oracle (direct per-term FP64 evaluation, all host cores) on a bounded sample of the
+    workload: strided (regime, r) rows with every class, the full lam grid and all samples."""
     from oracle import oracle as O
 
     threads = O.default_threads()
-    K, R, NL = w.K, len(w.r), len(w.lam)
-
-    def cells_for(rows):
-        ri = np.linspace(0, R - 1, rows).round().astype(np.int64)
-        kk, rr, ll = np.meshgrid(np.arange(K), ri, np.arange(NL), indexing="ij")
-        return np.zeros(kk.size, np.int32), kk.ravel(), rr.ravel(), ll.ravel()
-
-    cal = cells_for(1)
+    K, NL = w.K, len(w.lam)
+    cal, _ = oracle_rows(w, 1)
     t0 = time.perf_counter()
     O.eval_cells(w, *cal, threads=threads)
     t_cal = max(time.perf_counter() - t0, 1e-3)
-    rows = int(max(1, min(R, seconds / t_cal)))
-    cells = cells_for(rows)
+    rows = int(max(1, min(len(w.cp) * len(w.r), seconds / t_cal)))
+    cells, terms = oracle_rows(w, rows)
     t0 = time.perf_counter()
     O.eval_cells(w, *cells, threads=threads)
     dt = time.perf_counter() - t0
-    terms = int(rows * NL * int(w.N.sum()))
-    return {"value": terms / dt, "unit": UNIT, "cores": threads, "kind": "oracle",
-            "sample": f"{rows} strided r rows x {NL} lam x {K} classes x {int(w.N[0])} samples = {terms:.3e} terms, "
-                      f"direct per-term FP64 oracle, {dt:.2f} s wall"}, dt
+    return {"value": terms / dt, "unit": UNIT, "cores": threads, "cpu_model": cpu_model(), "kind": "oracle",
+            "sample": f"{rows} strided (regime, r) rows x {NL} lam x {K} classes x {int(w.N[0])} samples = "
+                      f"{terms:.3e} terms, direct per-term FP64 oracle, {dt:.2f} s wall"}, dt
 
 
 # ------------------------------------------------------------------ our implementation
@@ -230,7 +276,7 @@ def run_ours(args):
     dev = torch.device("cuda", local_rank)
     from paper_2607_16892_gb300 import kvdro as kv
 
-    w = lognormal_workload_k8_n1e5()
+    w = WORKLOADS[args.workload]()
     M, E, K, R, NL, F = len(w.cp), len(w.eps), w.K, len(w.r), len(w.lam), len(w.fractiles)
     terms = w.terms()
     ctx = kv.kvdro_create(local_rank)
@@ -290,12 +336,20 @@ def run_ours(args):
     # roofline of the grid kernel (this rank's launches)
     kernel_ms = statistics.mean(grid_ms)
     achieved = terms / (kernel_ms / 1e3)
-    peak = props.multi_processor_count * TERMS_PER_CLK_PER_SM * SM_MAX_MHZ_RECIPE * 1e6
+    sms = props.multi_processor_count
+    peak = sms * TERMS_PER_CLK_PER_SM * SM_MAX_MHZ_RECIPE * 1e6
+    peak_paper = sms * 128.0 / PAPER_FORM_LANE_OPS_PER_TERM * SM_MAX_MHZ_RECIPE * 1e6
+    traffic, inst_per_term = profile_figures()
     roofline = {"bound": "alu", "achieved": achieved, "peak": peak, "unit": UNIT, "frac": achieved / peak,
-                "traffic": profile_traffic(), "kernel": "k_grid<EXACT> (FP32 outputs)",
-                "kernel_ms_mean": kernel_ms,
-                "peak_basis": f"{props.multi_processor_count} SMs x ({FMA_TERMS_PER_CLK_PER_SM:.0f} terms/clk/SM on packed "
-                              f"FP32 adds + {ALU_TERMS_PER_CLK_PER_SM:.0f} on integer sad) x {SM_MAX_MHZ_RECIPE:.0f} MHz"}
+                "traffic": traffic, "kernel": "k_grid<EXACT> (FP32 outputs)",
+                "kernel_ms_mean": kernel_ms, "per_term_op": PER_TERM_OP,
+                "peak_basis": f"{sms} SMs x ({FMA_TERMS_PER_CLK_PER_SM:.0f} terms/clk/SM on packed "
+                              f"FP32 adds + {ALU_TERMS_PER_CLK_PER_SM:.0f} on integer sad) x {SM_MAX_MHZ_RECIPE:.0f} MHz",
+                "frac_survey_basis": achieved / peak_paper,
+                "survey_basis": f"{sms} SMs x 128 FP32 lanes / {PAPER_FORM_LANE_OPS_PER_TERM:.0f} lane-ops per term of "
+                                f"the 3-candidate phi (2 FMA, 2 max, 1 add) x {SM_MAX_MHZ_RECIPE:.0f} MHz = "
+                                f"{peak_paper:.4g} terms/s; the kernel does not do that work per term",
+                "inst_per_term": inst_per_term}
     if clocks.get("sm_mhz"):
         roofline["frac_at_sampled_clock"] = achieved / (peak * clocks["sm_mhz"] / SM_MAX_MHZ_RECIPE)
 
@@ -341,18 +395,15 @@ def run_ours(args):
 
 def run_reference(args):
     rank, _, world = dist_env()
-    w = lognormal_workload_k8_n1e5()
     if rank != 0:
         return
+    w = WORKLOADS[args.workload]()
     from oracle import oracle as O
 
     threads = O.default_threads()
-    K, R, NL = w.K, len(w.r), len(w.lam)
-    rows = 2  # per step: 2 strided r rows x all lam x all classes x all samples
-    ri = np.linspace(0, R - 1, rows).round().astype(np.int64)
-    kk, rr, ll = np.meshgrid(np.arange(K), ri, np.arange(NL), indexing="ij")
-    cells = (np.zeros(kk.size, np.int32), kk.ravel(), rr.ravel(), ll.ravel())
-    step_terms = rows * NL * int(w.N.sum())
+    K, NL = w.K, len(w.lam)
+    rows = 2  # per step: 2 strided (regime, r) rows x all lam x all classes x all samples
+    cells, step_terms = oracle_rows(w, rows)
     for _ in range(args.warmup):
         O.eval_cells(w, *cells, threads=threads)
     t0 = time.perf_counter()
@@ -360,14 +411,15 @@ def run_reference(args):
         O.eval_cells(w, *cells, threads=threads)
     dt = time.perf_counter() - t0
     value = step_terms * args.steps / dt
-    sample = (f"per step {rows} strided r rows x {NL} lam x {K} classes x {int(w.N[0])} samples = "
+    sample = (f"per step {rows} strided (regime, r) rows x {NL} lam x {K} classes x {int(w.N[0])} samples = "
               f"{step_terms:.3e} terms, direct per-term FP64 oracle")
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": workload_config(w, world),
-        "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle", "sample": sample},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "cpu_model": cpu_model(), "kind": "oracle",
+                         "sample": sample},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
@@ -494,36 +546,21 @@ def run_cpu_suite(args):
                           "sort_quantiles_s": t_sort, "samples": int(w.N.sum())}), flush=True)
 
 
-# BCD-DRO solve times of the paper's scalability table (Sec. 5.2; hardware unstated), by
-# (classes, configurations, samples per class): context for the host solve, not a target
-PAPER_BCD_SECONDS = {(3, 4, 100): 0.17, (4, 4, 150): 0.8, (5, 5, 200): 4.3, (6, 6, 300): 10.5, (8, 6, 500): 22.4,
-                     (10, 8, 1000): 81.2, (15, 12, 2000): 257.7}
-
-
-def run_bcd(args):
-    """Alg. 1 end to end on the scalability instances: the library's worst-case cost tables
-    (one exact-dual pass per support size) and the host blocks, each timed on the wall clock."""
-    from paper_2607_16892_gb300 import bcd
-    from synth import SCALABILITY_SIZES, bcd_instance
-
-    warm = bcd.Problem(**bcd_instance(2, 2, 50, 8, L_cap=64))
-    bcd.solve(warm, bcd.gpu_tables(warm))          # library load, CUDA context, scipy import
-    for I, K, N, J in SCALABILITY_SIZES:
-        p = bcd.Problem(**bcd_instance(I, K, N, J))
-        t0 = time.perf_counter()
-        tables = bcd.gpu_tables(p)
-        res = bcd.solve(p, tables)
-        total = time.perf_counter() - t0
-        sec = res.seconds
-        print(json.dumps({"bcd": True, "instance": p.name, "classes": I, "configs": K, "samples_per_class": N,
-                          "gpus_modelled": J, "configurations_in_Z": int(bcd.config_set(p.tau * p.pp, p.J).shape[0]),
-                          "total_s": total, "tables_s": sec["tables"], "lp1_s": sec["lp1"], "lp2_s": sec["lp2"],
-                          "block3_s": sec["block3"], "lp_rounds": res.lp_rounds,
-                          "outer_iterations": res.outer_iterations, "objective": res.objective,
-                          "admitted": float((p.arrival * res.pi.sum(axis=1)).sum() / p.arrival.sum()),
-                          "paper_bcd_s": PAPER_BCD_SECONDS.get((I, K, N)),
-                          "paper_note": "paper's BCD-DRO time, hardware unstated, LP over per-sample epigraph "
-                                        "variables; context only"}), flush=True)
+def case_workload(spec: str):
+    """The workload of a --case spec WORKLOAD:MODE[:key=val,...] and its mode (see --case)."""
+    parts = spec.split(":")
+    name, mode = parts[0], parts[1]
+    opts = dict(kv.split("=") for kv in parts[2].split(",")) if len(parts) > 2 and parts[2] else {}
+    w = WORKLOADS[name]()
+    if "m" in opts or "rstride" in opts:
+        regimes = np.arange(int(opts.get("m", len(w.cp))))
+        r_index = np.arange(0, len(w.r), int(opts.get("rstride", 1)))
+        w = slice_workload(w, regimes=regimes, r_index=r_index, name=w.name)
+    if "nl" in opts:
+        w.lam = np.logspace(np.log10(w.lam[0]), np.log10(w.lam[-1]), int(opts["nl"]))
+    if "L" in opts:  # a larger declared support: same samples, same grid
+        w.L = np.full(w.K, int(opts["L"]), np.int32)
+    return w, mode
 
 
 def run_case(args):
@@ -531,10 +568,8 @@ def run_case(args):
     import torch
 
     from paper_2607_16892_gb300 import kvdro as kv
-    from synth import WORKLOADS
 
-    name, mode = args.case.split(":")
-    w = WORKLOADS[name]()
+    w, mode = case_workload(args.case)
     dev = torch.device("cuda", 0)
     M, E, K, R, NL = len(w.cp), len(w.eps), w.K, len(w.r), len(w.lam)
     ctx = kv.kvdro_create(0)
@@ -550,8 +585,12 @@ def run_case(args):
             kv.kvdro_eval_grid(ctx, prec[mode], R, w.r, NL, w.lam, E, w.eps, M, w.cp, w.cw, r_idx=r_idx)
         torch.cuda.synchronize(dev)
         line = {"case": args.case, "run": i, "timed": i >= args.warmup, "wall_ms": 1e3 * (time.perf_counter() - t0)}
+        if mode not in ("sort", "dual", "envelope"):
+            line["terms"] = w.terms()
         if mode != "sort":
             line["kernel_ms"] = kv.kvdro_last_grid_ms(ctx)
+            if "terms" in line:
+                line["terms_per_s"] = w.terms() / (line["kernel_ms"] / 1e3)
         print(json.dumps(line), flush=True)
     kv.kvdro_destroy(ctx)
 
@@ -564,12 +603,8 @@ def main():
     if args.cpu_suite:
         run_cpu_suite(args)
         return
-    if args.bcd:
-        run_bcd(args)
-        return
     if args.suite:
         run_suite(args)
-        run_bcd(args)
         return
     if args.impl == "reference":
         run_reference(args)

@@ -71,8 +71,14 @@ typedef enum {
 /* Create a context on CUDA device `device_ordinal`.  *out receives the handle (NULL on error).
  * Two environment variables, read here, are test hooks and must not be set in production:
  * KVDRO_TEST_FAIL_ALLOC=n makes the context's n-th allocation fail (KVDRO_ENOMEM), and
- * KVDRO_TEST_SKIP_CHUNK=c makes the context's grid kernels leave staged chunk c uncopied with a
- * wait bound of about 1 ms, so every bounded wait on it runs out (KVDRO_ETIMEOUT). */
+ * KVDRO_TEST_SKIP_CHUNK=c makes this context's grid kernels leave staged chunk c uncopied with a
+ * wait bound of 1 ms, so every bounded wait on it runs out (KVDRO_ETIMEOUT).  The hook travels
+ * with this context's launches only; other contexts, on the same device or not, keep the
+ * production bound.
+ * Bounded waits: a grid kernel gives up waiting for a staged sample chunk only after 2 s of the
+ * GPU's global timer AND a minimum number of polls made while it was running, so a CTA that is
+ * descheduled (time-slicing, preemption) does not report a timeout on a copy that lands once it
+ * resumes. */
 int kvdro_create(kvdro_ctx** out, int device_ordinal);
 
 /*
@@ -175,8 +181,10 @@ int kvdro_last_grid_ms(kvdro_ctx* ctx, float* ms);
  * Arguments are those of kvdro_load_samples and kvdro_eval_grid with precision KVDRO_FP32,
  * on the current device, except that `lengths` and every output must be device memory, there
  * is no S output, and `err` (may be NULL) receives up to err_len bytes of error text.  The
- * call blocks until the samples' range check is read back; the outputs are written
- * asynchronously on `stream`.
+ * call works on `stream` and returns once the outputs are written (it reads the samples' range
+ * check and the kernels' status word back), so a grid kernel that gave up a bounded wait is
+ * reported here as KVDRO_ETIMEOUT (the outputs are then incomplete).  The test hook
+ * KVDRO_TEST_SKIP_CHUNK of kvdro_create is read at every call of this entry point.
  */
 #define KVDRO_NOALLOC_SCRATCH_BYTES (32u << 20)
 int kvdro_eval_grid_noalloc(int32_t K, const int64_t* offsets, const int32_t* lengths, const int32_t* L_max,

@@ -34,7 +34,7 @@ constexpr int32_t kMaxE = 64;
 constexpr int32_t kMaxM = 65536;
 constexpr int32_t kMaxF = 65536;
 constexpr int64_t kMaxKF = 1 << 22;
-constexpr long long kTestWaitCycles = 2000000;  // the wait test's bound: about 1 ms at 2 GHz
+constexpr long long kTestWaitNs = 1000000;  // the wait test's bound: 1 ms
 constexpr int32_t kMaxNLf32 = 256;
 constexpr int32_t kMaxNLf64 = 128;
 
@@ -190,6 +190,22 @@ int check_kernel_errors(kvdro_ctx* ctx, cudaStream_t s) {
         KV_CUDA(cudaMemsetAsync(static_cast<int32_t*>(ctx->errs.p) + 1, 0, sizeof(int32_t), s), "clearing status");
         return fail(ctx, KVDRO_ETIMEOUT, "a grid kernel gave up waiting for a staged sample chunk");
     }
+    return KVDRO_OK;
+}
+
+// Every r must lie in [L_in, L_in + L_max] of every class (the reservation domain of Sec. 2.2),
+// i.e. in [max_k L_in, min_k (L_in + L_max)]: O(R + K).
+int check_reservations(kvdro_ctx* ctx, int32_t R, const int32_t* r) {
+    int32_t k_lo = 0, k_hi = 0;
+    for (int32_t k = 1; k < ctx->K; k++) {
+        if (ctx->Lin[k] > ctx->Lin[k_lo]) k_lo = k;
+        if ((int64_t)ctx->Lin[k] + ctx->L[k] < (int64_t)ctx->Lin[k_hi] + ctx->L[k_hi]) k_hi = k;
+    }
+    const int64_t lo = ctx->Lin[k_lo], hi = (int64_t)ctx->Lin[k_hi] + ctx->L[k_hi];
+    for (int32_t i = 0; i < R; i++)
+        if ((int64_t)r[i] < lo || (int64_t)r[i] > hi)
+            return fail(ctx, KVDRO_EINVAL, "r[%d] = %d outside [L_in, L_in + L_max] of class %d", i, r[i],
+                        (int64_t)r[i] < lo ? k_lo : k_hi);
     return KVDRO_OK;
 }
 
@@ -456,10 +472,7 @@ int kvdro_eval_grid(kvdro_ctx* ctx, int precision, int32_t R, const int32_t* r, 
     if (!finite_nonneg(lam, NL)) return fail(ctx, KVDRO_EINVAL, "lam must be finite and >= 0");
     if (!finite_nonneg(eps, E)) return fail(ctx, KVDRO_EINVAL, "eps must be finite and >= 0");
     if (!finite_nonneg(c_p, M) || !finite_nonneg(c_w, M)) return fail(ctx, KVDRO_EINVAL, "costs must be finite and >= 0");
-    for (int32_t i = 0; i < R; i++)
-        for (int32_t k = 0; k < ctx->K; k++)
-            if ((int64_t)r[i] < ctx->Lin[k] || (int64_t)r[i] > (int64_t)ctx->Lin[k] + ctx->L[k])
-                return fail(ctx, KVDRO_EINVAL, "r[%d] = %d outside [L_in, L_in + L_max] of class %d", i, r[i], k);
+    if (int rc_ = check_reservations(ctx, R, r)) return rc_;
     const int64_t cells_out = (int64_t)M * E * ctx->K * R;
     const int64_t rows = (int64_t)M * E * ctx->K;
 
@@ -558,14 +571,13 @@ int kvdro_eval_grid(kvdro_ctx* ctx, int precision, int32_t R, const int32_t* r, 
     a.lam_idx_out = static_cast<int32_t*>(outs[2].dev);
     a.keys = static_cast<unsigned long long*>(ctx->keys.p);
     a.err = static_cast<int32_t*>(ctx->errs.p);
+    // Test hook of contexts created with KVDRO_TEST_SKIP_CHUNK: 1 ms waits that run out on one
+    // chunk.  It travels with this context's launches only.
+    a.test_skip_chunk = ctx->skip_chunk;
+    a.wait_ns = ctx->skip_chunk >= 0 ? kTestWaitNs : 0;
     const int64_t per_m = (int64_t)ctx->K * shape.r_blocks;
     const int64_t m_step = std::max<int64_t>(1, 0x7fffffffLL / per_m);
     ctx->grid_timed = false;
-    // Test hook: bounded waits of about 1 ms that run out on one chunk.  The setting lives in
-    // device globals, so while it is armed it applies to every grid launch of the process on this
-    // device; only contexts created with KVDRO_TEST_SKIP_CHUNK arm it, around their own launches.
-    if (ctx->skip_chunk >= 0)
-        KV_CUDA(kvdro::set_wait_test(ctx->skip_chunk, kTestWaitCycles, s), "arming the wait test");
     KV_CUDA(cudaEventRecord(ctx->grid_t0, s), "recording grid start");
     for (int64_t m0 = 0; m0 < M; m0 += m_step) {
         a.m0 = (int32_t)m0;
@@ -573,7 +585,6 @@ int kvdro_eval_grid(kvdro_ctx* ctx, int precision, int32_t R, const int32_t* r, 
         KV_CUDA(kvdro::launch_grid(KP, shape, a, s), "grid kernel");
     }
     KV_CUDA(cudaEventRecord(ctx->grid_t1, s), "recording grid end");
-    if (ctx->skip_chunk >= 0) KV_CUDA(kvdro::set_wait_test(-1, 0, s), "disarming the wait test");
     ctx->grid_timed = true;
 
     kvdro::FinalizeArgs fa;
@@ -616,10 +627,7 @@ int kvdro_eval_dual(kvdro_ctx* ctx, int32_t R, const int32_t* r, int32_t E, cons
     if (!r || !eps || !c_p || !c_w) return fail(ctx, KVDRO_EINVAL, "r, eps, c_p and c_w are required");
     if (!finite_nonneg(eps, E)) return fail(ctx, KVDRO_EINVAL, "eps must be finite and >= 0");
     if (!finite_nonneg(c_p, M) || !finite_nonneg(c_w, M)) return fail(ctx, KVDRO_EINVAL, "costs must be finite and >= 0");
-    for (int32_t i = 0; i < R; i++)
-        for (int32_t k = 0; k < ctx->K; k++)
-            if ((int64_t)r[i] < ctx->Lin[k] || (int64_t)r[i] > (int64_t)ctx->Lin[k] + ctx->L[k])
-                return fail(ctx, KVDRO_EINVAL, "r[%d] = %d outside [L_in, L_in + L_max] of class %d", i, r[i], k);
+    if (int rc_ = check_reservations(ctx, R, r)) return rc_;
     const int64_t cells = (int64_t)M * E * ctx->K * R;
     const int64_t rows = (int64_t)M * E * ctx->K;
     if (cells > 0x7fffffffLL * 256LL) return fail(ctx, KVDRO_EINVAL, "grid too large");

@@ -41,11 +41,16 @@ namespace {
 
 typedef unsigned long long u64;
 
-constexpr long long kWaitCycles = 4000000000LL;  // ~2 s at 2 GHz: bound on any barrier wait
-// The bound in force, and a test hook: a chunk index whose copy is never issued, so the waits
-// on its barrier run out (-1: none).  Set together by set_wait_test.
-__device__ long long g_wait_cycles = kWaitCycles;
-__device__ int g_test_skip_chunk = -1;
+// Bound on any barrier wait: 2 s of the GPU's global nanosecond timer, and at least
+// kWaitPollsPerNs polls per nanosecond of that bound spent polling (each poll suspends the
+// thread for at most kPollSuspendNs).  The timer keeps running while a CTA is descheduled
+// (time-slicing, preemption), but the poll count only grows while it runs, so a CTA that
+// was switched out for longer than the bound does not give up on a copy that lands soon
+// after it resumes.  kWaitPollCap bounds the loop even if the timer were to stop.
+constexpr long long kWaitNs = 2000000000LL;
+constexpr unsigned kPollSuspendNs = 1000;
+constexpr long long kWaitNsPerPoll = 4096;   // polls required: limit_ns / 4096
+constexpr unsigned kWaitPollCap = 1u << 28;
 
 constexpr int ilog2(int v) { return v <= 1 ? 0 : 1 + ilog2(v / 2); }
 
@@ -153,13 +158,38 @@ __device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
         : "memory");
     return ok != 0;
 }
+// The same test, suspending the thread for at most about `ns` nanoseconds while the phase is
+// incomplete.
+__device__ __forceinline__ bool mbar_try_for(uint32_t bar, uint32_t parity, uint32_t ns) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity), "r"(ns)
+        : "memory");
+    return ok != 0;
+}
+__device__ __forceinline__ unsigned long long global_ns() {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
 
-// Wait for phase `parity` of `bar`; gives up after g_wait_cycles and returns false.
-__device__ __noinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity) {
+// Wait for phase `parity` of `bar`.  Gives up and returns false once limit_ns nanoseconds of
+// the global timer have passed and the wait has polled at least limit_ns / kWaitNsPerPoll
+// times (or after kWaitPollCap polls in any case).  limit_ns <= 0 selects kWaitNs.
+__device__ __noinline__ bool mbar_wait_bounded(uint32_t bar, uint32_t parity, long long limit_ns) {
     if (mbar_try(bar, parity)) return true;
-    const long long t0 = clock64(), limit = g_wait_cycles;
-    while (!mbar_try(bar, parity)) {
-        if (clock64() - t0 > limit) return false;
+    if (limit_ns <= 0) limit_ns = kWaitNs;
+    const unsigned long long t0 = global_ns();
+    const unsigned min_polls = (unsigned)(limit_ns / kWaitNsPerPoll);
+    unsigned polls = 0;
+    while (!mbar_try_for(bar, parity, kPollSuspendNs)) {
+        ++polls;
+        if (polls >= kWaitPollCap) return false;
+        if (polls >= min_polls && (long long)(global_ns() - t0) > limit_ns) return false;
     }
     return true;
 }
@@ -283,7 +313,7 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
     const int nchunks = (int)((np + C::CHUNK - 1) / C::CHUNK);
     const float2* src = a.pairs + pbase;
     auto issue = [&](int c) {
-        if (c == g_test_skip_chunk) return;  // test hook: nothing will complete this chunk's barrier
+        if (c == a.test_skip_chunk) return;  // test hook: nothing will complete this chunk's barrier
         const int s = c % C::STAGES;
         const int64_t cnt = min((int64_t)C::CHUNK, np - (int64_t)c * C::CHUNK);
         tma_bulk_load(smem_u32(ring + (size_t)s * C::CHUNK), src + (int64_t)c * C::CHUNK, (uint32_t)(cnt * sizeof(float2)),
@@ -338,7 +368,7 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
         }
         for (int c = 0; c < nchunks; c++) {
             const int s = c % C::STAGES;
-            if (!mbar_wait_bounded(smem_u32(&full[s]), (uint32_t)((c / C::STAGES) & 1))) timeout = true;
+            if (!mbar_wait_bounded(smem_u32(&full[s]), (uint32_t)((c / C::STAGES) & 1), a.wait_ns)) timeout = true;
             if (!timeout) {
                 const int cnt = (int)min((int64_t)C::CHUNK, np - (int64_t)c * C::CHUNK);
                 const float4* q = reinterpret_cast<const float4*>(ring + (size_t)s * C::CHUNK);
@@ -405,7 +435,7 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
         }
         for (int c = 0; c < nchunks; c++) {
             const int s = c % C::STAGES;
-            if (!mbar_wait_bounded(smem_u32(&full[s]), (uint32_t)((c / C::STAGES) & 1))) timeout = true;
+            if (!mbar_wait_bounded(smem_u32(&full[s]), (uint32_t)((c / C::STAGES) & 1), a.wait_ns)) timeout = true;
             if (!timeout) {
                 const int cnt = (int)min((int64_t)C::CHUNK, np - (int64_t)c * C::CHUNK);
                 const float4* q = reinterpret_cast<const float4*>(ring + (size_t)s * C::CHUNK);
@@ -549,7 +579,7 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
         int pending = 0;  // loads since the last fold
         for (int c = 0; c < nchunks; c++) {
             const int s = c % C::STAGES;
-            if (!mbar_wait_bounded(smem_u32(&full[s]), (uint32_t)((c / C::STAGES) & 1))) timeout = true;
+            if (!mbar_wait_bounded(smem_u32(&full[s]), (uint32_t)((c / C::STAGES) & 1), a.wait_ns)) timeout = true;
             if (!timeout) {
                 const int cnt = (int)min((int64_t)C::CHUNK, np - (int64_t)c * C::CHUNK);
                 const float4* q = reinterpret_cast<const float4*>(ring + (size_t)s * C::CHUNK);
@@ -608,7 +638,7 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
         if (tid == 0) {
             atomicOr(a.err + 1, kErrTimeout);
             for (int c = consumed; c < issued; c++)
-                (void)mbar_wait_bounded(smem_u32(&full[c % C::STAGES]), (uint32_t)((c / C::STAGES) & 1));
+                (void)mbar_wait_bounded(smem_u32(&full[c % C::STAGES]), (uint32_t)((c / C::STAGES) & 1), a.wait_ns);
         }
         __syncthreads();
         return;
@@ -775,15 +805,6 @@ cudaError_t grid_prepare(Prec p) {
     cudaError_t e = cudaFuncSetAttribute(k_grid<CfgF32>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
     if (e != cudaSuccess) return e;
     return cudaFuncSetAttribute(k_grid<CfgF32Wide>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
-}
-
-cudaError_t set_wait_test(int skip_chunk, long long wait_cycles, cudaStream_t s) {
-    const long long w = wait_cycles > 0 ? wait_cycles : kWaitCycles;
-    cudaError_t e = cudaMemcpyToSymbolAsync(g_test_skip_chunk, &skip_chunk, sizeof(int), 0, cudaMemcpyHostToDevice, s);
-    if (e != cudaSuccess) return e;
-    e = cudaMemcpyToSymbolAsync(g_wait_cycles, &w, sizeof(long long), 0, cudaMemcpyHostToDevice, s);
-    if (e != cudaSuccess) return e;
-    return cudaStreamSynchronize(s);  // the host values are on this stack frame
 }
 
 cudaError_t launch_grid(Prec p, const GridShape& sh, GridArgs a, cudaStream_t s) {

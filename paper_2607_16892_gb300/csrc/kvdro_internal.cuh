@@ -85,6 +85,11 @@ struct GridArgs {
     int32_t* lam_idx_out;       // optional [M][E][K][R]
     unsigned long long* keys;   // [M][E][K] argmin keys (initialised to all ones)
     int32_t* err;               // [1] |= kErrTimeout
+    // Bounded waits and their test hook, per launch: wait_ns bounds each wait on a staged chunk
+    // (0: the default of about 2 s); test_skip_chunk >= 0 leaves that chunk's copy unissued, so
+    // the waits on it run out (-1 in production).
+    long long wait_ns;
+    int32_t test_skip_chunk;
 };
 
 struct FinalizeArgs {
@@ -115,9 +120,6 @@ GridShape grid_shape(Prec p, int32_t R, int32_t NL, int32_t E, int32_t max_L);  
 cudaError_t grid_prepare(Prec p);             // per-device attribute setup of every variant of p
 // Launches over regimes [a.m0, a.m0 + a.m_count); fills a.LT, a.RG, a.r_blocks from `sh`.
 cudaError_t launch_grid(Prec p, const GridShape& sh, GridArgs a, cudaStream_t s);
-// Test hook for the bounded waits of the grid kernel: skip_chunk >= 0 makes every CTA leave that
-// chunk's copy unissued, so its waits give up after wait_cycles; (-1, 0) restores the defaults.
-cudaError_t set_wait_test(int skip_chunk, long long wait_cycles, cudaStream_t s);
 cudaError_t launch_finalize(Prec p, const FinalizeArgs& a, cudaStream_t s);
 
 // dual.cu: exact minimisation over gamma >= 0 per (regime, radius, class, reservation)

@@ -7,7 +7,9 @@
 #include <cuda_runtime.h>
 
 #include <cmath>
+#include <cstdint>
 #include <cstdio>
+#include <cstdlib>
 #include <initializer_list>
 #include <mutex>
 
@@ -143,12 +145,18 @@ extern "C" int kvdro_eval_grid_noalloc(int32_t K, const int64_t* offsets, const 
     for (int32_t i = 0; i < M; i++)
         if (!std::isfinite(c_p[i]) || c_p[i] < 0 || !std::isfinite(c_w[i]) || c_w[i] < 0)
             return report(err, err_len, KVDRO_EINVAL, "costs must be finite and >= 0");
-    for (int32_t i = 0; i < R; i++)
+    {
+        // every r must lie in [L_in, L_in + L_max] of every class: in [max L_in, min (L_in + L_max)]
+        int64_t lo = 0, hi = INT64_MAX;
         for (int32_t k = 0; k < K; k++) {
             const int64_t lin = L_in ? L_in[k] : 0;
-            if (r[i] < lin || (int64_t)r[i] > lin + L_max[k])
-                return report(err, err_len, KVDRO_EINVAL, "r outside [L_in, L_in + L_max] of some class");
+            lo = lin > lo ? lin : lo;
+            hi = lin + L_max[k] < hi ? lin + L_max[k] : hi;
         }
+        for (int32_t i = 0; i < R; i++)
+            if ((int64_t)r[i] < lo || (int64_t)r[i] > hi)
+                return report(err, err_len, KVDRO_EINVAL, "r outside [L_in, L_in + L_max] of some class");
+    }
     if (!device_pointer(lengths)) return report(err, err_len, KVDRO_EINVAL, "lengths must be device memory");
     for (const void* o : {(const void*)cost, (const void*)lam_idx, (const void*)r_idx, (const void*)min_cost,
                           (const void*)fhat})
@@ -294,6 +302,14 @@ extern "C" int kvdro_eval_grid_noalloc(int32_t K, const int64_t* offsets, const 
     a.lam_idx_out = lam_idx;
     a.keys = reinterpret_cast<unsigned long long*>(S + o_keys);
     a.err = sa.err;
+    // The bounded-wait test hook, read at every call (see kvdro_create): a 1 ms bound and one
+    // chunk left uncopied, so the waits on it run out.
+    a.test_skip_chunk = -1;
+    a.wait_ns = 0;
+    if (const char* f = std::getenv("KVDRO_TEST_SKIP_CHUNK")) {
+        a.test_skip_chunk = std::atoi(f);
+        a.wait_ns = 1000000;
+    }
     const int64_t per_m = (int64_t)K * shape.r_blocks;
     const int64_t m_step = per_m > 0x7fffffffLL ? 1 : 0x7fffffffLL / per_m;
     for (int64_t m0 = 0; m0 < M; m0 += m_step) {
@@ -317,6 +333,14 @@ extern "C" int kvdro_eval_grid_noalloc(int32_t K, const int64_t* offsets, const 
     fa.min_cost = min_cost;
     fa.fhat = fhat;
     if (r_idx || min_cost || fhat) NA_CUDA(kvdro::launch_finalize(kvdro::Prec::F32, fa, s));
+    // A grid CTA that gave up a bounded wait wrote none of its cells, so the outputs are
+    // incomplete: report it here (the next call clears the status word).
+    int32_t status = 0;
+    NA_CUDA(cudaMemcpyAsync(&status, S + o_err + sizeof(int32_t), sizeof(int32_t), cudaMemcpyDeviceToHost, s));
+    NA_CUDA(cudaStreamSynchronize(s));
+    if (status & kvdro::kErrTimeout)
+        return report(err, err_len, KVDRO_ETIMEOUT,
+                      "a grid kernel gave up waiting for a staged sample chunk; the outputs are incomplete");
 #undef NA_CUDA
     return KVDRO_OK;
 }

@@ -136,6 +136,32 @@ def _stream(s: Any):
     raise TypeError(f"unsupported stream {type(s)}")
 
 
+def _numel(a: Any) -> int:
+    if isinstance(a, np.ndarray):
+        return int(a.size)
+    if hasattr(a, "numel"):
+        return int(a.numel())
+    return int(np.asarray(a).size)
+
+
+def _need(name: str, a: Any, n: int) -> None:
+    """Raise ValueError unless array ``a`` (if given) holds exactly ``n`` elements: the library
+    reads or writes exactly that many through the pointer, so a shorter buffer would be
+    overrun (on the device or on the host)."""
+    if a is not None and _numel(a) != n:
+        raise ValueError(f"{name} has {_numel(a)} elements; the call needs exactly {n}")
+
+
+def _on_device(name: str, a: Any) -> None:
+    if a is not None and not (hasattr(a, "is_cuda") and a.is_cuda):
+        raise ValueError(f"{name} must be a CUDA tensor")
+
+
+# Class count and sample total of each context's loaded samples (keyed by the handle), so
+# that outputs sized by them can be checked before a call.
+_loaded: dict = {}
+
+
 def _check(ctx, status: int):
     if status != KVDRO_OK:
         msg = load_library().kvdro_last_error(ctx).decode() if ctx else ""
@@ -153,17 +179,57 @@ def kvdro_create(device_ordinal: int = 0) -> ctypes.c_void_p:
     return h
 
 
+def _check_samples(K: int, off: np.ndarray, lengths, lm: np.ndarray, li) -> None:
+    if int(K) < 1:
+        raise ValueError(f"K = {K} must be at least 1")
+    _need("offsets", off, int(K) + 1)
+    _need("L_max", lm, int(K))
+    _need("L_in", li, int(K))
+    _need("lengths", lengths, int(off[-1]))
+
+
 def kvdro_load_samples(ctx, K: int, offsets, lengths, L_max, L_in=None, stream=None) -> None:
     off = _host(offsets, np.int64)
     lm = _host(L_max, np.int32)
     li = None if L_in is None else _host(L_in, np.int32)
+    _check_samples(K, off, lengths, lm, li)
+    key = getattr(ctx, "value", ctx)
+    _loaded.pop(key, None)
     _check(ctx, load_library().kvdro_load_samples(ctx, int(K), off.ctypes.data, _ptr(lengths, np.int32), lm.ctypes.data,
                                                   None if li is None else li.ctypes.data, _stream(stream)))
+    _loaded[key] = (int(K), int(off[-1]))
+
+
+def _ctx_K(ctx):
+    """Class count of the context's loaded samples (None if unknown here)."""
+    got = _loaded.get(getattr(ctx, "value", ctx))
+    return None if got is None else got[0]
 
 
 def kvdro_quantiles(ctx, F: int, fractiles, out, stream=None) -> None:
     fr = _host(fractiles, np.float64)
+    _need("fractiles", fr, int(F))
+    K = _ctx_K(ctx)
+    if K is not None:
+        _need("out", out, K * int(F))
     _check(ctx, load_library().kvdro_quantiles(ctx, int(F), fr.ctypes.data, _ptr(out, np.int32), _stream(stream)))
+
+
+def _check_grid(R, rr, E, ee, M, cp, cw, NL=None, ll=None) -> None:
+    _need("r", rr, int(R))
+    if NL is not None:
+        _need("lam", ll, int(NL))
+    _need("eps", ee, int(E))
+    _need("c_p", cp, int(M))
+    _need("c_w", cw, int(M))
+
+
+def _check_outputs(K: int, R: int, E: int, M: int, NL=None, **outs) -> None:
+    rows = M * E * K
+    size = {"S": M * K * R * (NL or 0), "cost": rows * R, "lam_idx": rows * R, "gamma": rows * R, "r_idx": rows,
+            "min_cost": rows, "fhat": rows}
+    for name, a in outs.items():
+        _need(name, a, size[name])
 
 
 def kvdro_eval_grid(ctx, precision: int, R: int, r, NL: int, lam, E: int, eps, M: int, c_p, c_w, S=None, cost=None,
@@ -171,6 +237,11 @@ def kvdro_eval_grid(ctx, precision: int, R: int, r, NL: int, lam, E: int, eps, M
     ft = np.float32 if precision == KVDRO_FP32 else np.float64
     rr, ll, ee = _host(r, np.int32), _host(lam, np.float64), _host(eps, np.float64)
     cp, cw = _host(c_p, np.float64), _host(c_w, np.float64)
+    _check_grid(R, rr, E, ee, M, cp, cw, NL=NL, ll=ll)
+    K = _ctx_K(ctx)
+    if K is not None:
+        _check_outputs(K, int(R), int(E), int(M), NL=int(NL), S=S, cost=cost, lam_idx=lam_idx, r_idx=r_idx,
+                       min_cost=min_cost, fhat=fhat)
     _check(ctx, load_library().kvdro_eval_grid(
         ctx, int(precision), int(R), rr.ctypes.data, int(NL), ll.ctypes.data, int(E), ee.ctypes.data, int(M),
         cp.ctypes.data, cw.ctypes.data, _ptr(S, ft), _ptr(cost, ft), _ptr(lam_idx, np.int32), _ptr(r_idx, np.int32),
@@ -181,6 +252,10 @@ def kvdro_eval_dual(ctx, R: int, r, E: int, eps, M: int, c_p, c_w, cost=None, ga
                     min_cost=None, fhat=None, stream=None) -> None:
     rr, ee = _host(r, np.int32), _host(eps, np.float64)
     cp, cw = _host(c_p, np.float64), _host(c_w, np.float64)
+    _check_grid(R, rr, E, ee, M, cp, cw)
+    K = _ctx_K(ctx)
+    if K is not None:
+        _check_outputs(K, int(R), int(E), int(M), cost=cost, gamma=gamma, r_idx=r_idx, min_cost=min_cost, fhat=fhat)
     _check(ctx, load_library().kvdro_eval_dual(
         ctx, int(R), rr.ctypes.data, int(E), ee.ctypes.data, int(M), cp.ctypes.data, cw.ctypes.data,
         _ptr(cost, np.float64), _ptr(gamma, np.float64), _ptr(r_idx, np.int32), _ptr(min_cost, np.float64),
@@ -188,6 +263,9 @@ def kvdro_eval_dual(ctx, R: int, r, E: int, eps, M: int, c_p, c_w, cost=None, ga
 
 
 def kvdro_sorted_samples(ctx, out, stream=None) -> None:
+    got = _loaded.get(getattr(ctx, "value", ctx))
+    if got is not None:
+        _need("out", out, got[1])
     _check(ctx, load_library().kvdro_sorted_samples(ctx, _ptr(out, np.int32), _stream(stream)))
 
 
@@ -206,6 +284,13 @@ def kvdro_eval_grid_noalloc(K: int, offsets, lengths, L_max, L_in, R: int, r, NL
     li = None if L_in is None else _host(L_in, np.int32)
     rr, ll, ee = _host(r, np.int32), _host(lam, np.float64), _host(eps, np.float64)
     cp, cw = _host(c_p, np.float64), _host(c_w, np.float64)
+    _check_samples(K, off, lengths, lm, li)
+    _check_grid(R, rr, E, ee, M, cp, cw, NL=NL, ll=ll)
+    _check_outputs(int(K), int(R), int(E), int(M), cost=cost, lam_idx=lam_idx, r_idx=r_idx, min_cost=min_cost,
+                   fhat=fhat)
+    for name, a in (("lengths", lengths), ("cost", cost), ("lam_idx", lam_idx), ("r_idx", r_idx),
+                    ("min_cost", min_cost), ("fhat", fhat)):
+        _on_device(name, a)
     buf = ctypes.create_string_buffer(512)
     st = load_library().kvdro_eval_grid_noalloc(
         int(K), off.ctypes.data, _ptr(lengths, np.int32), lm.ctypes.data, None if li is None else li.ctypes.data,
@@ -226,4 +311,5 @@ def kvdro_last_error(ctx) -> str:
 
 def kvdro_destroy(ctx) -> None:
     if ctx:
+        _loaded.pop(getattr(ctx, "value", ctx), None)
         load_library().kvdro_destroy(ctx)

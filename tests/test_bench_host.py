@@ -6,6 +6,7 @@ import os
 import subprocess
 import sys
 
+import numpy as np
 import pytest
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
@@ -91,10 +92,27 @@ def test_reference_arm_line_has_the_contract_keys():
 
 def test_stale_profile_is_not_reported(tmp_path, monkeypatch):
     prof = tmp_path / "p.md"
-    prof.write_text("grid_cu_sha256: " + "0" * 64 + "\ntraffic_bytes_per_launch: 123\n")
+    prof.write_text("grid_cu_sha256: " + "0" * 64 + "\ntraffic_bytes_per_launch: 123\ninst_per_term: 1.1\n")
     monkeypatch.setattr(bench, "PROFILE", str(prof))
-    assert bench.profile_traffic() is None
+    assert bench.profile_figures() == (None, None)
     import hashlib
     h = hashlib.sha256(open(bench.GRID_SOURCE, "rb").read()).hexdigest()
-    prof.write_text(f"grid_cu_sha256: {h}\ntraffic_bytes_per_launch: 123\n")
-    assert bench.profile_traffic() == 123.0
+    prof.write_text(f"grid_cu_sha256: {h}\ntraffic_bytes_per_launch: 123\ninst_per_term: 1.1\n")
+    assert bench.profile_figures() == (123.0, 1.1)
+
+
+def test_oracle_sample_rows_stride_over_regimes_and_reservations():
+    """The CPU-baseline sample: strided (regime, r) rows, each with every class and lam value."""
+    from synth import regime_sweep_workload_k8_n2e5
+    w = regime_sweep_workload_k8_n2e5()
+    (m, k, r, l), terms = bench.oracle_rows(w, 4)
+    M, K, R, NL = len(w.cp), w.K, len(w.r), len(w.lam)
+    assert m.size == 4 * K * NL and terms == 4 * NL * int(w.N.sum())
+    assert m[0] == 0 and r[0] == 0 and m[-1] == M - 1 and r[-1] == R - 1
+    assert set(np.unique(k)) == set(range(K)) and set(np.unique(l)) == set(range(NL))
+
+
+def test_case_spec_options():
+    w, mode = bench.case_workload("regimes_k8_n2e5:fp32:m=16,nl=256,L=4194305,rstride=4")
+    assert mode == "fp32" and len(w.cp) == 16 and len(w.lam) == 256 and len(w.r) == 512
+    assert (w.L == 4194305).all() and w.lam[0] == 1e-3 and abs(w.lam[-1] - 1e3) < 1e-9

@@ -2,9 +2,13 @@
 
 The envelope evaluator of the oracle (the same finite sum regrouped by affine pieces over
 exact cumulative counts, pinned in test_oracle_pins.py) gives every cell of the full grids;
-the direct per-term evaluator checks randomly drawn cells of the same runs.  The 8-class
-workload runs exactly as bench.py times it (FP32, all outputs), plus an FP64 slice.
+the direct per-term evaluator checks randomly drawn cells of the same runs.  The regime
+sweep (all 1024 regimes) runs exactly as bench.py times it (FP32, the same outputs); the
+8-class workload runs in FP32, exact and native FP64 over its full grid.
 """
+
+import os
+from concurrent.futures import ThreadPoolExecutor
 
 import numpy as np
 import pytest
@@ -70,11 +74,13 @@ def test_heavy_tail_k16_n1e6_exact_full_grid():
     print(rep)
 
 
-def test_lognormal_k8_n1e5_fp64_slice():
-    w = slice_workload(lognormal_workload_k8_n1e5(), r_index=np.arange(3, 4096, 16), name="k8_fp64_slice")
+def test_lognormal_k8_n1e5_fp64_full_grid():
+    """Native FP64 arithmetic per term on every cell of the 8-class grid (4096 r x 128 lam)."""
+    w = lognormal_workload_k8_n1e5()
     gpu = run(w, kvdro.KVDRO_FP64)
-    compare_full(w, gpu, oracle_from_S(w, O.envelope_grid(w)), "fp64")
-    direct_cells(w, gpu["S"], 1024, RTOL["fp64"], 2)
+    rep = compare_full(w, gpu, oracle_from_S(w, O.envelope_grid(w)), "fp64")
+    rep["direct"] = direct_cells(w, gpu["S"], 1024, RTOL["fp64"], 2)
+    print(rep)
 
 
 def test_heavy_tail_k16_n1e6_fp32_full_grid():
@@ -94,24 +100,54 @@ def test_regime_sweep_slice_and_critical_fractile():
     ora = oracle_from_S(w, O.envelope_grid(w))
     compare_full(w, gpu, ora, "fp32")
     direct_cells(w, gpu["S"], 256, RTOL["fp32"], 4)
-    # eps = 0 (index 0): the oracle's argmin is the grid point at or next to each regime's
-    # critical-fractile quantile (Prop. "Critical Fractile Structure"); the GPU's choice is that
-    # point too, or one whose oracle cost ties with it within the FP32 tolerance.
+    _critical_fractile_rows(w, gpu["r_idx"], ora["cost"], ora["r_idx"], RTOL["fp32"])
+
+
+def _critical_fractile_rows(w, gpu_r_idx, ora_cost, ora_r_idx, rtol):
+    """eps = 0 (index 0): the oracle's argmin is the grid point at or next to each regime's
+    critical-fractile quantile q = c_p / (c_p + c_w) (Prop. "Critical Fractile Structure"); the
+    GPU's choice is that point too, or one whose oracle cost ties with it within rtol."""
     q = O.quantiles(w, w.cp / (w.cp + w.cw))  # [k, m]
-    rtol = RTOL["fp32"]
     for mm in range(len(w.cp)):
         for k in range(w.K):
             lo = w.r[np.searchsorted(w.r, q[k, mm], side="right") - 1] if q[k, mm] >= w.r[0] else w.r[0]
             hi = w.r[min(np.searchsorted(w.r, q[k, mm], side="left"), len(w.r) - 1)]
-            r_ora = w.r[ora["r_idx"][mm, 0, k]]
+            r_ora = w.r[ora_r_idx[mm, 0, k]]
             assert lo <= r_ora <= hi, (mm, k, r_ora, q[k, mm])
-            g = gpu["r_idx"][mm, 0, k]
+            g = gpu_r_idx[mm, 0, k]
             if not lo <= w.r[g] <= hi:
-                row = ora["cost"][mm, 0, k]
+                row = ora_cost[mm, 0, k]
                 assert row[g] <= row.min() * (1 + rtol), (mm, k, w.r[g], q[k, mm])
 
 
-@pytest.mark.parametrize("iteration", [0, 1])
+def test_regime_sweep_all_1024_regimes_as_benchmarked():
+    """Every (regime, radius, class, r) of the regime sweep (8 classes x 200,000 samples, 2048 r,
+    64 lam, 16 eps, 1024 cost ratios), run exactly as bench.py times it: cost, lam index, r index,
+    minimum cost and F-hat against the oracle's envelope sums and eps epilogue, computed 16 regimes
+    at a time on all host cores; the critical fractile at eps = 0 on every regime; quantiles."""
+    w = regime_sweep_workload_k8_n2e5()
+    gpu = run(w, kvdro.KVDRO_FP32, outputs=("cost", "lam_idx", "r_idx", "min_cost", "fhat", "quant"))
+    assert np.array_equal(gpu["quant"], O.quantiles(w, w.fractiles))
+    rtol = RTOL["fp32"]
+    M = len(w.cp)
+    step = 16
+
+    def chunk(m0):
+        mi = np.arange(m0, min(M, m0 + step))
+        wc = slice_workload(w, regimes=mi, name=f"regimes_{m0}")
+        ora = oracle_from_S(wc, O.envelope_grid(wc, threads=1))
+        sub = {key: gpu[key][mi] for key in ("cost", "lam_idx", "r_idx", "min_cost", "fhat")}
+        rep = compare_full(wc, sub, ora, "fp32")
+        _critical_fractile_rows(wc, sub["r_idx"], ora["cost"], ora["r_idx"], rtol)
+        return rep
+
+    with ThreadPoolExecutor(max(1, min(16, os.cpu_count() or 1))) as ex:
+        reps = list(ex.map(chunk, range(0, M, step)))
+    print({"cost_max_rel": max(r["cost_max_rel"] for r in reps), "r_idx_exact": sum(r["r_idx_exact"] for r in reps),
+           "lam_idx_exact": sum(r["lam_idx_exact"] for r in reps)})
+
+
+@pytest.mark.parametrize("iteration", [0, 25, 49])
 def test_drift_loop_k32_n1e6_iteration(iteration):
     w = drift_loop_workload_k32_n1e6(iteration)
     gpu = run(w, kvdro.KVDRO_FP32)

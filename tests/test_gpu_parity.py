@@ -242,6 +242,41 @@ def test_a_wait_that_runs_out_reports_etimeout_and_the_device_stays_usable(monke
     compare_full(w, run(w, P[prec]), O.solve(w), prec)  # a context without the hook, same device
 
 
+def test_the_wait_hook_of_one_context_leaves_another_on_the_same_device_unaffected(monkeypatch):
+    """The bounded-wait test hook travels with one context's launches: while a hooked context's
+    grid kernels give up on their never-copied chunk (device outputs, so the call returns at
+    once), a second context on the same device, on another stream, evaluates correctly, and the
+    hooked context still reports KVDRO_ETIMEOUT."""
+    rng = np.random.default_rng(4)
+    w = make([rng.integers(0, 900, 20000), rng.integers(0, 1000, 9000)], 1000, np.arange(0, 1001, 37),
+             np.logspace(-2, 1.5, 24), [0.0, 10.0, 90.0], [10.0, 2.0], [1.0, 1.0])
+    monkeypatch.setenv("KVDRO_TEST_SKIP_CHUNK", "1")
+    hooked = kvdro.kvdro_create(0)
+    monkeypatch.delenv("KVDRO_TEST_SKIP_CHUNK")
+    plain = kvdro.kvdro_create(0)
+    M, E, K, R, NL = len(w.cp), len(w.eps), w.K, len(w.r), len(w.lam)
+    s1, s2 = torch.cuda.Stream(), torch.cuda.Stream()
+    try:
+        d = torch.from_numpy(w.samples).cuda()
+        for ctx in (hooked, plain):
+            kvdro.kvdro_load_samples(ctx, w.K, w.offsets, d, w.L, w.L_in)
+        ev = lambda ctx, st, **kw: kvdro.kvdro_eval_grid(ctx, P["fp32"], R, w.r, NL, w.lam, E, w.eps, M, w.cp, w.cw,
+                                                         stream=st, **kw)
+        ref = O.solve(w)
+        for _ in range(2):
+            r_dev = torch.empty((M, E, K), dtype=torch.int32, device="cuda")
+            ev(hooked, s1, r_idx=r_dev)  # its CTAs now wait out their bound on stream s1
+            got = {"cost": np.empty((M, E, K, R), np.float32), "lam_idx": np.empty((M, E, K, R), np.int32),
+                   "r_idx": np.empty((M, E, K), np.int32), "min_cost": np.empty((M, E, K), np.float32)}
+            ev(plain, s2, **got)  # host outputs: returns once they are filled
+            compare_full(w, got, ref, "fp32")
+            assert _status(kvdro.kvdro_sync, plain) == kvdro.KVDRO_OK
+            assert _status(kvdro.kvdro_sync, hooked) == kvdro.KVDRO_ETIMEOUT
+    finally:
+        kvdro.kvdro_destroy(hooked)
+        kvdro.kvdro_destroy(plain)
+
+
 def test_exact_mode_rejects_support_above_its_limit():
     ctx = kvdro.kvdro_create(0)
     try:

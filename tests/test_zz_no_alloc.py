@@ -1,17 +1,21 @@
-"""kvdro_eval_grid_noalloc against kvdro_eval_grid, through the C ABI, on two calls in a row.
+"""kvdro_eval_grid_noalloc against kvdro_eval_grid and against the CPU oracle, through the C ABI.
 
 The no-allocation entry point serves callers that cannot allocate device memory when they
 need a reservation answer (for example a serving engine whose free memory all belongs to its
 KV-cache pool).  It must give the same results as the context-based entry point, also when
-the previous call left other data in its shared static scratch.  This file is collected last
-so that a stop-at-first-failure run has already run every other test.
+the previous call left other data in its shared static scratch, and the oracle's results
+within the FP32 tolerance, for every kernel it can choose (the exact kernel with packed and
+integer columns up to a support of 2^19, the all-integer one up to 2^22, the FP32-arithmetic
+one above).  This file is collected last so that a stop-at-first-failure run has already run
+every other test.
 """
 
 import numpy as np
 import pytest
 
-from synth import random_case, lognormal_workload_k3_n1e3
-from tests.parity import RTOL, check_argmin, rel_close
+from oracle import oracle as O
+from synth import Workload, random_case, lognormal_workload_k3_n1e3
+from tests.parity import RTOL, check_argmin, compare_full, rel_close
 
 torch = pytest.importorskip("torch")
 pytestmark = pytest.mark.gpu
@@ -78,3 +82,51 @@ def test_noalloc_rejects_a_problem_larger_than_its_scratch():
         kvdro.kvdro_eval_grid_noalloc(1, np.array([0, n]), samples, [1000], None, len(w.r), w.r, len(w.lam), w.lam,
                                       1, w.eps[:1], 1, w.cp[:1], w.cw[:1], r_idx=r_idx)
     assert e.value.status == kvdro.KVDRO_EINVAL and "static scratch" in str(e.value)
+
+
+def _classes_on(L, K, seed, n=(3000, 400)):
+    """K (1 or 2) classes on the support [0, L], with samples at both ends, and a small grid.
+    The static scratch holds 4 bytes per support point and class, so supports above 2^21
+    take one class."""
+    rng = np.random.default_rng(seed)
+    cls = [np.concatenate([[0, L], rng.integers(0, L + 1, n[0])]).astype(np.int32),
+           rng.integers(max(0, L - 5000), L + 1, n[1]).astype(np.int32)][:K]
+    off = np.concatenate([[0], np.cumsum([c.size for c in cls])]).astype(np.int64)
+    return Workload(name=f"classes_L{L}", samples=np.concatenate(cls), offsets=off,
+                    L=np.full(K, L, np.int32), L_in=np.zeros(K, np.int32),
+                    r=np.array([0, 1, L // 3, L - 1, L], np.int32), lam=np.logspace(-3, 2, 23),
+                    eps=np.array([0.0, 700.0]), cp=np.array([10.0, 0.5]), cw=np.array([1.0, 3.0]),
+                    fractiles=np.array([0.5]))
+
+
+def test_noalloc_matches_the_oracle():
+    """Against the CPU oracle (direct per-term sums, eps epilogue, argmin), not another GPU path."""
+    w = random_case(303, K=3, N=(4100, 515, 37), L=(2500, 2500, 2500), R=41, n_lam=33, n_eps=3, M=2,
+                    lam_range=(1e-3, 100.0), eps_max=200.0)
+    rep = compare_full(w, _noalloc(w), O.solve(w), "fp32")
+    assert rep["r_idx_exact"] > 0
+
+
+@pytest.mark.parametrize("L,K", [((1 << 20) + 3, 2), ((1 << 22) + 4096, 1)])
+def test_noalloc_large_supports_match_the_oracle(L, K):
+    """A support in (2^19, 2^22] takes the all-integer exact kernel; one above 2^22 the
+    FP32-arithmetic kernel.  Both through the static scratch, against the oracle."""
+    w = _classes_on(L, K, 44 + K)
+    compare_full(w, _noalloc(w), O.solve(w), "fp32")
+
+
+def test_noalloc_reports_a_wait_that_runs_out(monkeypatch):
+    """With the bounded-wait test hook set, every grid CTA gives up on the chunk whose copy is
+    never issued; the call returns KVDRO_ETIMEOUT (its outputs are incomplete) instead of
+    KVDRO_OK, and the next call without the hook is correct."""
+    rng = np.random.default_rng(5)
+    cls = rng.integers(0, 900, 20000).astype(np.int32)  # five staged chunks
+    w = Workload(name="wait", samples=cls, offsets=np.array([0, cls.size], np.int64), L=np.array([1000], np.int32),
+                 L_in=np.zeros(1, np.int32), r=np.array([10, 200, 600], np.int32), lam=np.array([0.5, 5.0]),
+                 eps=np.array([0.0, 10.0]), cp=np.array([10.0]), cw=np.array([1.0]), fractiles=np.array([0.5]))
+    monkeypatch.setenv("KVDRO_TEST_SKIP_CHUNK", "2")
+    with pytest.raises(kvdro.KvdroError) as e:
+        _noalloc(w)
+    assert e.value.status == kvdro.KVDRO_ETIMEOUT and "gave up waiting" in str(e.value)
+    monkeypatch.delenv("KVDRO_TEST_SKIP_CHUNK")
+    compare_full(w, _noalloc(w), O.solve(w), "fp32")
