@@ -154,7 +154,11 @@ def test_invalid_arguments_are_rejected_on_the_host():
         ev = lambda **kw: kvdro.kvdro_eval_grid(ctx, kvdro.KVDRO_FP32, 1, [1], 1, [1.0], 1, [0.0], 1, [2.0], [1.0], **kw)
         assert _status(ev) == kvdro.KVDRO_ESTATE  # nothing loaded yet
         s = torch.tensor([1, 2, 3], dtype=torch.int32, device="cuda")
-        assert _status(kvdro.kvdro_load_samples, ctx, 0, np.array([0]), s, np.array([], np.int32)) == kvdro.KVDRO_EINVAL
+        with pytest.raises(ValueError):  # the binding rejects K = 0 before calling the library ...
+            kvdro.kvdro_load_samples(ctx, 0, np.array([0]), s, np.array([], np.int32))
+        off0 = np.array([0], np.int64)  # ... and so does the C ABI on its own
+        assert kvdro.load_library().kvdro_load_samples(ctx, 0, off0.ctypes.data, s.data_ptr(), None, None,
+                                                       None) == kvdro.KVDRO_EINVAL
         assert _status(kvdro.kvdro_load_samples, ctx, 1, np.array([1, 3]), s, np.array([10])) == kvdro.KVDRO_EINVAL
         assert _status(kvdro.kvdro_load_samples, ctx, 2, np.array([0, 0, 3]), s, np.array([10, 10])) == kvdro.KVDRO_EINVAL
         assert _status(kvdro.kvdro_load_samples, ctx, 1, np.array([0, 3]), s, np.array([0])) == kvdro.KVDRO_EINVAL
