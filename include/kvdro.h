@@ -175,8 +175,9 @@ int kvdro_last_grid_ms(kvdro_ctx* ctx, float* ms);
  * Calls share the array: it keeps the last call's contents (the call clears what must start at
  * zero), and calls whose GPU work overlaps in time race on it -- serialise them, e.g. on one
  * stream.  A problem whose scratch would exceed the array (about 12 bytes per sample plus
- * 4 bytes per support point and 8 bytes per (regime, radius, class) row) is rejected with
- * KVDRO_EINVAL and a message.
+ * 4 bytes per support point and 8 bytes per (regime, radius, class) row, and with more than 128
+ * lam values 12 bytes per (regime, radius, class, r) cell) is rejected with KVDRO_EINVAL and a
+ * message.
  *
  * Arguments are those of kvdro_load_samples and kvdro_eval_grid with precision KVDRO_FP32,
  * on the current device, except that `lengths` and every output must be device memory, there

@@ -36,6 +36,7 @@ constexpr int32_t kMaxF = 65536;
 constexpr int64_t kMaxKF = 1 << 22;
 constexpr long long kTestWaitNs = 1000000;  // the wait test's bound: 1 ms
 constexpr int32_t kMaxNLf32 = 256;
+constexpr int64_t kPartBytes = 256LL << 20;  // cap of the running-minimum buffer of lam blocks
 constexpr int32_t kMaxNLf64 = 128;
 
 struct Buf {
@@ -59,7 +60,7 @@ struct kvdro_ctx {
     std::vector<int64_t> off, pair_off, hist_off, N;
     std::vector<int32_t> L, Lin, hist_blocks, exp_blocks;
 
-    Buf sorted, pairs, hist, csum, sumx, meta, errs, in_stage, grid_in, keys, cost64, out_stage, ranks, scan_tot;
+    Buf sorted, pairs, hist, csum, sumx, meta, errs, in_stage, grid_in, keys, cost64, out_stage, ranks, scan_tot, part;
     void* pin = nullptr;  // pinned host staging
     size_t pin_bytes = 0;
     cudaEvent_t pin_free = nullptr;  // completes when the last copy out of `pin` is done
@@ -253,7 +254,7 @@ int kvdro_destroy(kvdro_ctx* ctx) {
     if (ctx->last_stream) cudaStreamSynchronize(ctx->last_stream);
     cudaDeviceSynchronize();
     for (Buf* b : {&ctx->sorted, &ctx->scan_tot, &ctx->pairs, &ctx->hist, &ctx->csum, &ctx->sumx, &ctx->meta, &ctx->errs, &ctx->in_stage,
-                   &ctx->grid_in, &ctx->keys, &ctx->cost64, &ctx->out_stage, &ctx->ranks})
+                   &ctx->grid_in, &ctx->keys, &ctx->cost64, &ctx->out_stage, &ctx->ranks, &ctx->part})
         release(*b);
     if (ctx->pin) cudaFreeHost(ctx->pin);
     if (ctx->pin_free) cudaEventDestroy(ctx->pin_free);
@@ -481,8 +482,14 @@ int kvdro_eval_grid(kvdro_ctx* ctx, int precision, int32_t R, const int32_t* r, 
     if (!g.ok) return fail(ctx, KVDRO_ECUDA, "cannot select device %d", ctx->device);
     ctx->last_stream = s;
 
-    // Launch shape: lam tiles x r groups of warps per CTA.
-    const kvdro::GridShape shape = kvdro::grid_shape(KP, R, NL, E, max_L);
+    // Launch shape: lam tiles x r groups of warps per CTA.  The exact kernel takes at most
+    // kExactLamBlock lam values per launch; a larger grid runs as consecutive launches over blocks
+    // of it (the last block may be smaller and take its own shape).
+    const int32_t lam_blk = KP == Prec::EXACT ? kvdro::kExactLamBlock : NL;
+    const int32_t nblk = (NL + lam_blk - 1) / lam_blk;
+    const int32_t NL_last = NL - (nblk - 1) * lam_blk;
+    const kvdro::GridShape shape = kvdro::grid_shape(KP, R, std::min(NL, lam_blk), E, max_L);
+    const kvdro::GridShape shape_last = kvdro::grid_shape(KP, R, NL_last, E, max_L);
 
     // Grid parameters in one upload.
     const size_t gbytes = align_up((size_t)R * 4, 8) + 8 * ((size_t)NL + E + 2 * (size_t)M);
@@ -575,14 +582,36 @@ int kvdro_eval_grid(kvdro_ctx* ctx, int precision, int32_t R, const int32_t* r, 
     // chunk.  It travels with this context's launches only.
     a.test_skip_chunk = ctx->skip_chunk;
     a.wait_ns = ctx->skip_chunk >= 0 ? kTestWaitNs : 0;
-    const int64_t per_m = (int64_t)ctx->K * shape.r_blocks;
-    const int64_t m_step = std::max<int64_t>(1, 0x7fffffffLL / per_m);
+    a.lam0 = 0;
+    a.NL_out = NL;
+    a.part_val = nullptr;
+    a.part_idx = nullptr;
+    a.part_first = a.part_last = 1;
+    const int64_t per_m = (int64_t)ctx->K * std::max(shape.r_blocks, shape_last.r_blocks);
+    int64_t m_step = std::max<int64_t>(1, 0x7fffffffLL / per_m);
+    if (nblk > 1) {
+        // the running minimum over lam blocks, 12 bytes per (regime, eps, class, r), for at most
+        // kPartBytes worth of regimes at a time
+        const int64_t per_regime = (int64_t)E * ctx->K * R * 12;
+        m_step = std::max<int64_t>(1, std::min<int64_t>(m_step, kPartBytes / per_regime));
+        const int64_t cells = std::min<int64_t>(m_step, M) * (per_regime / 12);
+        if ((rc = ensure(ctx, ctx->part, (size_t)cells * 12))) return rc;
+        a.part_val = static_cast<double*>(ctx->part.p);
+        a.part_idx = reinterpret_cast<int32_t*>(static_cast<char*>(ctx->part.p) + (size_t)cells * 8);
+    }
     ctx->grid_timed = false;
     KV_CUDA(cudaEventRecord(ctx->grid_t0, s), "recording grid start");
     for (int64_t m0 = 0; m0 < M; m0 += m_step) {
         a.m0 = (int32_t)m0;
         a.m_count = (int32_t)std::min<int64_t>(m_step, M - m0);
-        KV_CUDA(kvdro::launch_grid(KP, shape, a, s), "grid kernel");
+        for (int32_t b = 0; b < nblk; b++) {
+            a.lam = d_lam + (size_t)b * lam_blk;
+            a.NL = b + 1 < nblk ? lam_blk : NL_last;
+            a.lam0 = b * lam_blk;
+            a.part_first = b == 0;
+            a.part_last = b + 1 == nblk;
+            KV_CUDA(kvdro::launch_grid(KP, b + 1 < nblk ? shape : shape_last, a, s), "grid kernel");
+        }
     }
     KV_CUDA(cudaEventRecord(ctx->grid_t1, s), "recording grid end");
     ctx->grid_timed = true;

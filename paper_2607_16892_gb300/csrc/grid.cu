@@ -75,8 +75,8 @@ struct GridCfg {
     static_assert(FLUSH >= 0 && UNROLL >= 1 && FCOLS >= 0 && FCOLS <= TL, "shape parameters out of range");
 };
 // 2 r x 8 lam tiles, up to 16 warps per CTA and (FP32, exact) two CTAs per SM (64 registers)
-// for up to 128 lam values; for 129..256 lam values the exact kernel runs one CTA of up to 32
-// such warps per SM and the FP32 kernel 2 x 16 tiles.  FP64: 2 x 8 tiles.
+// for up to 128 lam values; larger lam grids run the exact kernel in blocks of 128 lam values
+// (kExactLamBlock), and the FP32 kernel takes 2 x 16 tiles.  FP64: 2 x 8 tiles.
 // All stage 4096-sample chunks (32 KB) through a 2-deep ring.  The FP32 variants fold their
 // partial sums every 2 chunks (256 samples per lane); the exact variants fold as often as their
 // support size requires.  The narrow FP32 variant unrolls the sample loop 8 times, the exact
@@ -86,13 +86,13 @@ using CfgF32 = GridCfg<Prec::F32, 2, 8, 2, 2, 512, 4096, 2, 8>;
 using CfgF32Wide = GridCfg<Prec::F32, 2, 16, 2, 1, 512, 4096, 2, 2>;
 using CfgF64 = GridCfg<Prec::F64, 2, 8, 0, 1, 512, 4096, 2>;
 using CfgExact = GridCfg<Prec::EXACT, 2, 8, 0, 2, 512, 4096, 2, 4>;
-using CfgExactWide = GridCfg<Prec::EXACT, 2, 8, 0, 1, 1024, 4096, 2, 4>;
 // Above a support of 2^19 the packed FP32 sums (exact only up to 2^24) would fold every few loads;
 // there every column takes the integer absolute differences, whose sums fold far less often.
 using CfgExactInt = GridCfg<Prec::EXACT, 2, 8, 0, 2, 512, 4096, 2, 8, 0>;
-using CfgExactIntWide = GridCfg<Prec::EXACT, 2, 8, 0, 1, 1024, 4096, 2, 8, 0>;
 constexpr int32_t kExactIntAboveL = 1 << 19;
 constexpr int kWarpsTarget = 16;  // warps per CTA the r groups fill up to
+static_assert(kExactLamBlock == kWarpsTarget * CfgExact::TL && kExactLamBlock == kWarpsTarget * CfgExactInt::TL,
+              "one launch of the exact kernel takes 16 warps of lam tiles");
 
 // ---------------------------------------------------------------- PTX helpers
 
@@ -265,6 +265,19 @@ __device__ __forceinline__ void cta_epilogue(const GridArgs& a, const double* s_
         if (lane == 0) {
             const size_t row = ((size_t)m * a.E + e) * a.K + k;
             const size_t o = row * a.R + ri;
+            bj += a.lam0;
+            if (a.part_val) {  // lam blocks: merge with the earlier blocks (they hold lower indices)
+                const size_t q = ((((size_t)(m - a.m0)) * a.E + e) * a.K + k) * a.R + ri;
+                if (!a.part_first && !(best < a.part_val[q])) {
+                    best = a.part_val[q];
+                    bj = a.part_idx[q];
+                }
+                if (!a.part_last) {
+                    a.part_val[q] = best;
+                    a.part_idx[q] = bj;
+                    continue;
+                }
+            }
             u64 key;
             if constexpr (F32OUT) {
                 const float cf = (float)best;
@@ -669,7 +682,7 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
             const double S = tot * s_inv_n;
             s_S[(r_local0 + i) * NLpad + lj] = S;
             if (a.S_out) {
-                const size_t o = (((size_t)m * a.K + k) * a.R + ri) * a.NL + lj;
+                const size_t o = (((size_t)m * a.K + k) * a.R + ri) * a.NL_out + a.lam0 + lj;
                 if (P == Prec::F32 || a.f32_out) static_cast<float*>(a.S_out)[o] = (float)S;
                 else static_cast<double*>(a.S_out)[o] = S;
             }
@@ -722,7 +735,7 @@ __global__ void __launch_bounds__(kEnvThreads) k_envelope(const GridArgs a) {
         const double tot = branch_sum(cp, cw, mu, nu, (double)Lk, eta, N, cnt, below_s, (int64_t)Lk * cnt - sx);
         const double S = tot * inv_n;
         s_S[rl * a.NL + j] = S;
-        if (a.S_out) static_cast<double*>(a.S_out)[(((size_t)m * a.K + k) * a.R + ri) * a.NL + j] = S;
+        if (a.S_out) static_cast<double*>(a.S_out)[(((size_t)m * a.K + k) * a.R + ri) * a.NL_out + a.lam0 + j] = S;
     }
     __syncthreads();
     cta_epilogue<false>(a, s_S, s_lam, s_eps, a.NL, kEnvR, r_cta0, m, k);
@@ -778,11 +791,9 @@ GridShape grid_shape(Prec p, int32_t R, int32_t NL, int32_t E, int32_t max_L) {
         return sh;
     }
     if (p == Prec::F64) return shape_for<CfgF64>(2, R, NL, E);
-    if (p == Prec::EXACT) {
-        const bool narrow = NL <= kWarpsTarget * CfgExact::TL;
-        if (max_L > kExactIntAboveL)
-            return narrow ? shape_for<CfgExactInt>(6, R, NL, E) : shape_for<CfgExactIntWide>(7, R, NL, E);
-        return narrow ? shape_for<CfgExact>(3, R, NL, E) : shape_for<CfgExactWide>(5, R, NL, E);
+    if (p == Prec::EXACT) {  // NL <= kExactLamBlock: larger grids launch in blocks
+        if (max_L > kExactIntAboveL) return shape_for<CfgExactInt>(6, R, NL, E);
+        return shape_for<CfgExact>(3, R, NL, E);
     }
     if (NL <= kWarpsTarget * CfgF32::TL) return shape_for<CfgF32>(0, R, NL, E);
     return shape_for<CfgF32Wide>(1, R, NL, E);
@@ -794,9 +805,7 @@ cudaError_t grid_prepare(Prec p) {
     if (p == Prec::F64) return cudaFuncSetAttribute(k_grid<CfgF64>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
     if (p == Prec::EXACT) {
         cudaError_t e = cudaFuncSetAttribute(k_grid<CfgExact>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
-        if (e == cudaSuccess) e = cudaFuncSetAttribute(k_grid<CfgExactWide>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
         if (e == cudaSuccess) e = cudaFuncSetAttribute(k_grid<CfgExactInt>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
-        if (e == cudaSuccess) e = cudaFuncSetAttribute(k_grid<CfgExactIntWide>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
         return e;
     }
     if (p == Prec::ENVELOPE)
@@ -816,9 +825,7 @@ cudaError_t launch_grid(Prec p, const GridShape& sh, GridArgs a, cudaStream_t s)
     if (p == Prec::ENVELOPE) k_envelope<<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
     else if (p == Prec::F64) k_grid<CfgF64><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
     else if (p == Prec::EXACT && sh.variant == 3) k_grid<CfgExact><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
-    else if (p == Prec::EXACT && sh.variant == 5) k_grid<CfgExactWide><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
-    else if (p == Prec::EXACT && sh.variant == 6) k_grid<CfgExactInt><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
-    else if (p == Prec::EXACT) k_grid<CfgExactIntWide><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
+    else if (p == Prec::EXACT) k_grid<CfgExactInt><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
     else if (sh.variant == 0) k_grid<CfgF32><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
     else k_grid<CfgF32Wide><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
     return cudaGetLastError();

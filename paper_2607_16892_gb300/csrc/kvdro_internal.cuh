@@ -90,7 +90,20 @@ struct GridArgs {
     // the waits on it run out (-1 in production).
     long long wait_ns;
     int32_t test_skip_chunk;
+    // Lam blocks: a grid of more lam values than one launch takes runs as consecutive launches over
+    // blocks of it (ascending lam).  lam / NL are this block's values; lam0 is the index of its
+    // first value in the caller's grid of NL_out values.  With several blocks, part_val / part_idx
+    // ([m - m0][E][K][R]) carry each (r, eps) pair's minimum over the earlier blocks; the first
+    // block starts them, the last writes the outputs.  One block: part_val is null, lam0 = 0.
+    int32_t lam0, NL_out;
+    double* part_val;
+    int32_t* part_idx;
+    int32_t part_first, part_last;
 };
+
+// The largest lam grid one launch of the exact kernel takes (16 warps of 2 x 8 tiles); larger
+// grids run in blocks of it.
+constexpr int32_t kExactLamBlock = 128;
 
 struct FinalizeArgs {
     const unsigned long long* keys;

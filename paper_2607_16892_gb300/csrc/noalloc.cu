@@ -183,6 +183,16 @@ extern "C" int kvdro_eval_grid_noalloc(int32_t K, const int64_t* offsets, const 
     const size_t o_sorted = take((size_t)total * 4);
     const size_t o_pairs = take((size_t)pair_total * 8);
     const size_t o_keys = take((size_t)rows * 8);
+    // more lam values than one launch of the exact kernel takes: the running minimum over lam blocks
+    const bool exact_ok = [&] {
+        for (int32_t k = 0; k < K; k++)
+            if (L_max[k] > kvdro::kExactMaxL) return false;
+        return true;
+    }();
+    const int32_t lam_blk = exact_ok ? kvdro::kExactLamBlock : NL;
+    const int32_t nblk = (NL + lam_blk - 1) / lam_blk;
+    const size_t part_cells = nblk > 1 ? (size_t)rows * R : 0;
+    const size_t o_part_val = take(part_cells * 8), o_part_idx = take(part_cells * 4);
     const int64_t scan_tiles = (max_bins + kvdro::scan_tile_bins() - 1) / kvdro::scan_tile_bins();
     const size_t o_tiles = take((size_t)K * scan_tiles * 16);
     if (o > (size_t)KVDRO_NOALLOC_SCRATCH_BYTES) {
@@ -268,14 +278,12 @@ extern "C" int kvdro_eval_grid_noalloc(int32_t K, const int64_t* offsets, const 
 
     // ---- the grid kernel (the exact one, FP32 outputs, whenever every support is at most 2^22;
     // else the FP32-arithmetic one) and the argmin finalisation
-    bool exact_ok = true;
     int32_t max_L = 0;
-    for (int32_t k = 0; k < K; k++) {
-        exact_ok = exact_ok && L_max[k] <= kvdro::kExactMaxL;
-        max_L = L_max[k] > max_L ? L_max[k] : max_L;
-    }
+    for (int32_t k = 0; k < K; k++) max_L = L_max[k] > max_L ? L_max[k] : max_L;
     const kvdro::Prec kp = exact_ok ? kvdro::Prec::EXACT : kvdro::Prec::F32;
-    const kvdro::GridShape shape = kvdro::grid_shape(kp, R, NL, E, max_L);
+    const int32_t NL_last = NL - (nblk - 1) * lam_blk;
+    const kvdro::GridShape shape = kvdro::grid_shape(kp, R, NL < lam_blk ? NL : lam_blk, E, max_L);
+    const kvdro::GridShape shape_last = kvdro::grid_shape(kp, R, NL_last, E, max_L);
     kvdro::GridArgs a;
     a.pairs = sa.pairs;
     a.pair_off = sa.pair_off;
@@ -310,12 +318,28 @@ extern "C" int kvdro_eval_grid_noalloc(int32_t K, const int64_t* offsets, const 
         a.test_skip_chunk = std::atoi(f);
         a.wait_ns = 1000000;
     }
-    const int64_t per_m = (int64_t)K * shape.r_blocks;
-    const int64_t m_step = per_m > 0x7fffffffLL ? 1 : 0x7fffffffLL / per_m;
+    a.lam0 = 0;
+    a.NL_out = NL;
+    a.part_val = nblk > 1 ? reinterpret_cast<double*>(S + o_part_val) : nullptr;
+    a.part_idx = nblk > 1 ? reinterpret_cast<int32_t*>(S + o_part_idx) : nullptr;
+    const double* d_lam = a.lam;
+    const int64_t per_m = (int64_t)K * (shape.r_blocks > shape_last.r_blocks ? shape.r_blocks : shape_last.r_blocks);
+    // one launch per lam block covers every regime (the running minimum holds all of them), so
+    // with lam blocks the regimes are not split
+    const int64_t m_step = nblk > 1 ? M : (per_m > 0x7fffffffLL ? 1 : 0x7fffffffLL / per_m);
+    if (nblk > 1 && per_m * M > 0x7fffffffLL)
+        return report(err, err_len, KVDRO_EINVAL, "too many CTAs for one launch over every regime");
     for (int64_t m0 = 0; m0 < M; m0 += m_step) {
         a.m0 = (int32_t)m0;
         a.m_count = (int32_t)(m_step < M - m0 ? m_step : M - m0);
-        NA_CUDA(kvdro::launch_grid(kp, shape, a, s));
+        for (int32_t b = 0; b < nblk; b++) {
+            a.lam = d_lam + (size_t)b * lam_blk;
+            a.NL = b + 1 < nblk ? lam_blk : NL_last;
+            a.lam0 = b * lam_blk;
+            a.part_first = b == 0;
+            a.part_last = b + 1 == nblk;
+            NA_CUDA(kvdro::launch_grid(kp, b + 1 < nblk ? shape : shape_last, a, s));
+        }
     }
     kvdro::FinalizeArgs fa;
     fa.keys = a.keys;
