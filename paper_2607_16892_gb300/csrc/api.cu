@@ -60,7 +60,8 @@ struct kvdro_ctx {
     std::vector<int64_t> off, pair_off, hist_off, N;
     std::vector<int32_t> L, Lin, hist_blocks, exp_blocks;
 
-    Buf sorted, pairs, hist, csum, sumx, meta, errs, in_stage, grid_in, keys, cost64, out_stage, ranks, scan_tot, part;
+    Buf sorted, pairs, hist, csum, sumx, meta, errs, in_stage, grid_in, keys, cost64, out_stage, ranks, scan_tot, part,
+        tile_lo;
     void* pin = nullptr;  // pinned host staging
     size_t pin_bytes = 0;
     cudaEvent_t pin_free = nullptr;  // completes when the last copy out of `pin` is done
@@ -254,7 +255,7 @@ int kvdro_destroy(kvdro_ctx* ctx) {
     if (ctx->last_stream) cudaStreamSynchronize(ctx->last_stream);
     cudaDeviceSynchronize();
     for (Buf* b : {&ctx->sorted, &ctx->scan_tot, &ctx->pairs, &ctx->hist, &ctx->csum, &ctx->sumx, &ctx->meta, &ctx->errs, &ctx->in_stage,
-                   &ctx->grid_in, &ctx->keys, &ctx->cost64, &ctx->out_stage, &ctx->ranks, &ctx->part})
+                   &ctx->grid_in, &ctx->keys, &ctx->cost64, &ctx->out_stage, &ctx->ranks, &ctx->part, &ctx->tile_lo})
         release(*b);
     if (ctx->pin) cudaFreeHost(ctx->pin);
     if (ctx->pin_free) cudaEventDestroy(ctx->pin_free);
@@ -313,6 +314,9 @@ int kvdro_load_samples(kvdro_ctx* ctx, int32_t K, const int64_t* offsets, const 
         ctx->hist_blocks[k + 1] = (int32_t)hb;
         ctx->exp_blocks[k + 1] = (int32_t)eb;
     }
+    // histogram blocks sized to fill whole waves of this device (the bound above still holds:
+    // no class gets more blocks than samples)
+    KV_CUDA(kvdro::hist_block_prefix(ctx->N.data(), K, ctx->hist_blocks.data()), "sizing the histogram");
     ctx->total = offsets[K];
     ctx->pair_total = ctx->pair_off[K];
     ctx->hist_total = ctx->hist_off[K];
@@ -328,6 +332,7 @@ int kvdro_load_samples(kvdro_ctx* ctx, int32_t K, const int64_t* offsets, const 
     for (int32_t k = 0; k < K; k++) max_bins = std::max<int64_t>(max_bins, (int64_t)L_max[k] + 1);
     const int64_t scan_tiles = (max_bins + kvdro::scan_tile_bins() - 1) / kvdro::scan_tile_bins();
     if ((rc = ensure(ctx, ctx->scan_tot, (size_t)K * scan_tiles * 16))) return rc;
+    if ((rc = ensure(ctx, ctx->tile_lo, ((size_t)ctx->exp_blocks[K] + K) * 4))) return rc;
     const size_t meta_bytes = (size_t)(K + 1) * 8 * 3 + (size_t)K * 8 + (size_t)K * 4 * 2 + (size_t)(K + 1) * 4 * 2 + 64;
     if ((rc = ensure(ctx, ctx->meta, meta_bytes))) return rc;
 
@@ -379,6 +384,7 @@ int kvdro_load_samples(kvdro_ctx* ctx, int32_t K, const int64_t* offsets, const 
     a.pairs = static_cast<float2*>(ctx->pairs.p);
     a.err = static_cast<int32_t*>(ctx->errs.p);
     a.tile_tot = static_cast<int64_t*>(ctx->scan_tot.p);
+    a.tile_lo = static_cast<int32_t*>(ctx->tile_lo.p);
     a.scan_tiles = (int32_t)scan_tiles;
     a.K = K;
     KV_CUDA(kvdro::launch_histogram(a, ctx->hist_blocks[K], s), "histogram kernel");

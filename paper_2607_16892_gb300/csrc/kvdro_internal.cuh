@@ -32,11 +32,15 @@ struct SortArgs {
     float2* pairs;              // [pair_off[K]]
     int32_t* err;               // [0] += out-of-range samples
     int64_t* tile_tot;          // [K][scan_tiles][2] scan tile totals (count, sum of v h[v])
+    int32_t* tile_lo;           // [exp_blocks[K] + K] per class from exp_blocks[k] + k: the bin of the
+                                // first position of each expansion tile, then the bin of position N - 1
     int32_t scan_tiles;         // scan tiles of the largest class: ceil((max L + 1) / scan tile bins)
     int32_t K;
 };
 
 // Launchers (sort.cu)
+// prefix[K + 1] of histogram blocks per class, sized to the current device (sort.cu)
+cudaError_t hist_block_prefix(const int64_t* N, int32_t K, int32_t* prefix);
 cudaError_t launch_histogram(const SortArgs& a, int32_t nblocks, cudaStream_t s);
 cudaError_t launch_scan(const SortArgs& a, cudaStream_t s);
 cudaError_t launch_expand(const SortArgs& a, int32_t nblocks, cudaStream_t s);

@@ -195,6 +195,7 @@ extern "C" int kvdro_eval_grid_noalloc(int32_t K, const int64_t* offsets, const 
     const size_t o_part_val = take(part_cells * 8), o_part_idx = take(part_cells * 4);
     const int64_t scan_tiles = (max_bins + kvdro::scan_tile_bins() - 1) / kvdro::scan_tile_bins();
     const size_t o_tiles = take((size_t)K * scan_tiles * 16);
+    const size_t o_tile_lo = take(((size_t)exp_blocks + K) * 4);
     if (o > (size_t)KVDRO_NOALLOC_SCRATCH_BYTES) {
         char msg[200];
         snprintf(msg, sizeof(msg), "the problem needs %zu bytes of scratch; the static scratch holds %zu bytes", o,
@@ -266,6 +267,7 @@ extern "C" int kvdro_eval_grid_noalloc(int32_t K, const int64_t* offsets, const 
     sa.pairs = reinterpret_cast<float2*>(S + o_pairs);
     sa.err = reinterpret_cast<int32_t*>(S + o_err);
     sa.tile_tot = reinterpret_cast<int64_t*>(S + o_tiles);
+    sa.tile_lo = reinterpret_cast<int32_t*>(S + o_tile_lo);
     sa.scan_tiles = (int32_t)scan_tiles;
     sa.K = K;
     NA_CUDA(kvdro::launch_histogram(sa, (int32_t)hist_blocks, s));

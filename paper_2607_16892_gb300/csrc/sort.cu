@@ -2,10 +2,14 @@
 // quantile gather.  The samples are their own sort keys and are bounded by L_k, so class k's
 // sorted order is fully determined by its histogram over [0, L_k]: histogram -> inclusive scan
 // (the cumulative count C[v] = #{x <= v}, i.e. N times the empirical CDF) -> expansion of every
-// output position p into the smallest v with C[v] > p.  The expansion also writes the (x', x')
-// float pairs that the grid kernel streams (x' = x plus the class's staging offset), NaN-padded
-// to a multiple of kPadSamples per class.
+// output position p into the smallest v with C[v] > p.  The scan also records, for every tile of
+// kExpandTile output positions, the bin its first position falls in; the expansion then marks
+// where each bin's run of positions starts inside the tile and takes a running maximum, O(N + L)
+// in all.  It also writes the (x', x') float pairs that the grid kernel streams (x' = x plus the
+// class's staging offset), NaN-padded to a multiple of kPadSamples per class.
 #include <math.h>
+
+#include <algorithm>
 
 #include "kvdro_internal.cuh"
 
@@ -20,7 +24,9 @@ constexpr int64_t kScanTile = (int64_t)kScanThreads * 4;  // bins per scan block
 constexpr int kExpandThreads = 512;
 constexpr int kExpandPerThread = 8;
 constexpr int64_t kExpandTile = (int64_t)kExpandThreads * kExpandPerThread;
-constexpr int kExpandCoarse = 2048;  // entries of the per-block coarse index of cumulative counts (8 KB)
+// Histogram slices get at least this many samples, so that counting outweighs clearing and
+// flushing the block's shared bins.
+constexpr int64_t kHistMinSlice = kHistSmemBins;
 
 __device__ __forceinline__ int find_segment(const int32_t* prefix, int K, int b) {
     // largest k with prefix[k] <= b; prefix is strictly increasing, prefix[0] = 0
@@ -37,9 +43,12 @@ __global__ void __launch_bounds__(kHistThreads) k_histogram(SortArgs a) {
     __shared__ int32_t sh_bad[kHistThreads / 32];
     __shared__ unsigned long long sh_sum[kHistThreads / 32];
     const int k = find_segment(a.hist_blocks, a.K, blockIdx.x);
+    // the class's samples in equal slices, one per block (at most kHistSlice each)
+    const int64_t nblk = a.hist_blocks[k + 1] - a.hist_blocks[k];
+    const int64_t slice_len = (a.offsets[k + 1] - a.offsets[k] + nblk - 1) / nblk;
     const int64_t slice = blockIdx.x - a.hist_blocks[k];
-    const int64_t beg = a.offsets[k] + slice * kHistSlice;
-    const int64_t end = min(a.offsets[k + 1], beg + kHistSlice);
+    const int64_t beg = a.offsets[k] + slice * slice_len;
+    const int64_t end = min(a.offsets[k + 1], beg + slice_len);
     const int32_t Lk = a.L[k];
     const int nb = min(Lk + 1, kHistSmemBins);
     int32_t* gh = a.hist + a.hist_off[k];
@@ -57,8 +66,9 @@ __global__ void __launch_bounds__(kHistThreads) k_histogram(SortArgs a) {
         else atomicAdd(&gh[x], 1);
     };
     // 16-byte loads of four samples over the slice's aligned middle (alignment is taken from the
-    // address: `lengths` is the caller's pointer), two loads in flight per thread per step;
-    // the unaligned head and the tail one sample at a time.
+    // address: `lengths` is the caller's pointer): each thread loads its next two vectors before
+    // it counts the current two, so four loads are in flight while the atomics run; the unaligned
+    // head and the tail one sample at a time.
     const int32_t* src = a.lengths;
     const int64_t mis = (int64_t)((reinterpret_cast<uintptr_t>(src + beg) >> 2) & 3);
     const int64_t vbeg = min(end, beg + ((4 - mis) & 3));
@@ -66,15 +76,27 @@ __global__ void __launch_bounds__(kHistThreads) k_histogram(SortArgs a) {
     const int64_t vend = vbeg + 4 * nvec;
     for (int64_t i = beg + threadIdx.x; i < vbeg; i += blockDim.x) count(__ldg(src + i));
     const int4* v4 = reinterpret_cast<const int4*>(src + vbeg);
+    const int64_t bd = blockDim.x;
     int64_t q = threadIdx.x;
-    for (; q + (int64_t)blockDim.x < nvec; q += 2 * (int64_t)blockDim.x) {
-        const int4 u = __ldg(v4 + q), w = __ldg(v4 + q + blockDim.x);
+    int4 u = make_int4(0, 0, 0, 0), w = make_int4(0, 0, 0, 0);
+    bool hu = q < nvec, hw = q + bd < nvec;
+    if (hu) u = __ldg(v4 + q);
+    if (hw) w = __ldg(v4 + q + bd);
+    while (hu) {
+        const int64_t qn = q + 2 * bd;
+        const bool nu = qn < nvec, nw = qn + bd < nvec;
+        int4 u2 = make_int4(0, 0, 0, 0), w2 = make_int4(0, 0, 0, 0);
+        if (nu) u2 = __ldg(v4 + qn);
+        if (nw) w2 = __ldg(v4 + qn + bd);
         count(u.x); count(u.y); count(u.z); count(u.w);
-        count(w.x); count(w.y); count(w.z); count(w.w);
-    }
-    if (q < nvec) {
-        const int4 u = __ldg(v4 + q);
-        count(u.x); count(u.y); count(u.z); count(u.w);
+        if (hw) {
+            count(w.x); count(w.y); count(w.z); count(w.w);
+        }
+        u = u2;
+        w = w2;
+        hu = nu;
+        hw = nw;
+        q = qn;
     }
     for (int64_t i = vend + threadIdx.x; i < end; i += blockDim.x) count(__ldg(src + i));
     __syncthreads();
@@ -86,8 +108,8 @@ __global__ void __launch_bounds__(kHistThreads) k_histogram(SortArgs a) {
         bad += __shfl_xor_sync(0xffffffffu, bad, o);
         sum += __shfl_xor_sync(0xffffffffu, sum, o);
     }
-    const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
-    if (l == 0) { sh_bad[w] = bad; sh_sum[w] = sum; }
+    const int wid = threadIdx.x >> 5, l = threadIdx.x & 31;
+    if (l == 0) { sh_bad[wid] = bad; sh_sum[wid] = sum; }
     __syncthreads();
     if (threadIdx.x == 0) {
         int tb = 0;
@@ -214,91 +236,98 @@ __global__ void __launch_bounds__(kScanThreads) k_scan_apply(SortArgs a) {
     }
     int32_t total;
     const int32_t incl = block_inclusive_scan<int32_t>(t, warp_tot32, &total);
+    // For the expansion: tile_lo[q] = the bin holding position q * kExpandTile for each tile q of
+    // the class's sorted samples, and one more entry: the bin holding the last position, N - 1.
+    // Every position lies in exactly one bin's run [C[v] - h[v], C[v]), so each entry is written once.
+    const int64_t Nk = a.offsets[k + 1] - a.offsets[k];
+    const int64_t tiles = (Nk + kExpandTile - 1) / kExpandTile;
+    int32_t* tl = a.tile_lo + a.exp_blocks[k] + k;
 #pragma unroll
     for (int j = 0; j < 4; j++)
-        if (i0 + j < n) h[i0 + j] = (int32_t)(cc + incl - t + w[j]);
+        if (i0 + j < n) {
+            const int64_t hi = cc + incl - t + w[j], lo = hi - cnt[j];
+            h[i0 + j] = (int32_t)hi;
+            if (lo < hi) {
+                for (int64_t q = (lo + kExpandTile - 1) / kExpandTile; q * kExpandTile < hi && q < tiles; q++)
+                    tl[q] = (int32_t)(i0 + j);
+                if (lo <= Nk - 1 && Nk - 1 < hi) tl[tiles] = (int32_t)(i0 + j);
+            }
+        }
 }
 
 __global__ void __launch_bounds__(kExpandThreads) k_expand(SortArgs a) {
-    // A coarse index of the class's cumulative counts in shared memory: entry c is C at the end of
-    // bucket c (buckets of `stride` consecutive bins).  Each thread finds its first position's
-    // bucket there, then the bin inside the bucket in global memory (log2(stride) steps), and
-    // walks on for its next positions.  The warp then stores its 256 values lane-contiguously
-    // through shared memory (rows of 9 words: conflict-free), so every store is coalesced.
-    __shared__ int32_t sK[kExpandCoarse];
-    __shared__ int32_t sV[kExpandThreads / 32][32 * 9];
+    // One tile of kExpandTile output positions [p0, p0 + kExpandTile).  Its positions fall in the
+    // bins [tile_lo[q], tile_lo[q + 1]] (recorded by the scan).  The run of bin v starts at position
+    // C[v - 1]; marking each non-empty bin's run start inside the tile (and the first bin at the
+    // tile's first position) and taking the running maximum gives every position its value, since
+    // values ascend with position.  Stores are lane-contiguous (coalesced).
+    __shared__ int32_t sv[kExpandTile];
+    __shared__ int32_t s_wmax[kExpandThreads / 32];
     const int k = find_segment(a.exp_blocks, a.K, blockIdx.x);
-    const int64_t tile = blockIdx.x - a.exp_blocks[k];
+    const int64_t q = blockIdx.x - a.exp_blocks[k];
     const int64_t Nk = a.offsets[k + 1] - a.offsets[k];
     const int64_t padk = a.pair_off[k + 1] - a.pair_off[k];
     const int32_t* C = a.hist + a.hist_off[k];
     const int32_t Lk = a.L[k];
-    const int32_t stride = (int32_t)(((int64_t)Lk + kExpandCoarse) / kExpandCoarse);  // ceil((Lk + 1) / kExpandCoarse)
-    const int32_t ncoarse = (int32_t)(((int64_t)Lk + stride) / stride);                 // ceil((Lk + 1) / stride)
-    for (int c = threadIdx.x; c < ncoarse; c += blockDim.x)
-        sK[c] = __ldg(C + min((int64_t)Lk, (int64_t)(c + 1) * stride - 1));
-    __syncthreads();
-    const int lane = threadIdx.x & 31;
-    int32_t* wv = sV[threadIdx.x >> 5];
-    const int64_t p0 = tile * kExpandTile + (int64_t)threadIdx.x * kExpandPerThread;
-    if (p0 < Nk) {
-        // smallest bucket c with sK[c] > p0 (the last bucket ends at Lk and C[Lk] = Nk > p0)
-        int32_t lo = 0, hi = ncoarse - 1;
-        while (lo < hi) {
-            const int32_t mid = (lo + hi) >> 1;
-            if ((int64_t)sK[mid] > p0) hi = mid; else lo = mid + 1;
+    const int64_t p0 = q * kExpandTile;
+    const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+    const int64_t pend = min(Nk, p0 + kExpandTile);  // sample positions of this tile
+    if (p0 < Nk) {  // block-uniform
+        const int32_t* tl = a.tile_lo + a.exp_blocks[k] + k;
+        const int32_t v_lo = tl[q], v_hi = tl[q + 1];
+        for (int i = tid; i < kExpandTile; i += kExpandThreads) sv[i] = i == 0 ? v_lo : -1;
+        __syncthreads();
+        // a non-empty bin after v_lo starts its run after p0 (C[v - 1] >= C[v_lo] > p0)
+        for (int64_t v = (int64_t)v_lo + 1 + tid; v <= v_hi; v += kExpandThreads) {
+            const int32_t start = __ldg(C + v - 1);
+            if (__ldg(C + v) > start && start < pend) sv[start - p0] = (int32_t)v;
         }
-        // then the smallest v in the bucket with C[v] > p0 (C at the bucket's end is sK[lo] > p0)
-        int32_t a0 = lo * stride, b0 = (int32_t)min((int64_t)Lk, (int64_t)(lo + 1) * stride - 1);
-        while (a0 < b0) {
-            const int32_t mid = (a0 + b0) >> 1;
-            if ((int64_t)__ldg(C + mid) > p0) b0 = mid; else a0 = mid + 1;
-        }
-        int32_t v = a0;
+        __syncthreads();
+        // inclusive running maximum: kExpandPerThread consecutive entries per thread, then across
+        // the lanes of the warp and across the warps
+        int32_t m[kExpandPerThread], run = -1;
 #pragma unroll
         for (int j = 0; j < kExpandPerThread; j++) {
-            const int64_t p = p0 + j;
-            if (p < Nk && (int64_t)__ldg(C + v) <= p) {
-                // Galloping search for the next bin: doubling steps, then bisection.  Gaps between
-                // consecutive sorted values can span thousands of empty bins in a heavy tail.
-                int32_t base = v, step = 1;  // invariant: C[base] <= p
-                while (step <= Lk - base && (int64_t)__ldg(C + base + step) <= p) {
-                    base += step;
-                    step <<= 1;
-                }
-                int32_t a = min(base + 1, Lk), b2 = (step <= Lk - base) ? base + step : Lk;  // both <= Lk
-                while (a < b2) {
-                    const int32_t mid = (a + b2) >> 1;
-                    if ((int64_t)__ldg(C + mid) > p) b2 = mid; else a = mid + 1;
-                }
-                v = a;
-            }
-            wv[lane * 9 + j] = v;  // positions past Nk are never stored as samples
+            run = max(run, sv[tid * kExpandPerThread + j]);
+            m[j] = run;
         }
-    }
-    __syncwarp();
-    // lane-contiguous stores: position idx of the warp's 256 lives at wv[(idx / 8) * 9 + idx % 8]
-    const int64_t wbase = tile * kExpandTile + (int64_t)(threadIdx.x >> 5) * 32 * kExpandPerThread;
-    int32_t* out = a.sorted + a.offsets[k];
-    float2* pr = a.pairs + a.pair_off[k];
+        int32_t incl = run;
 #pragma unroll
-    for (int i = 0; i < kExpandPerThread; i++) {
-        const int idx = i * 32 + lane;
-        const int64_t p = wbase + idx;
-        if (p < Nk) out[p] = wv[(idx >> 3) * 9 + (idx & 7)];
+        for (int o = 1; o < 32; o <<= 1) {
+            const int32_t y = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl = max(incl, y);
+        }
+        if (lane == 31) s_wmax[wid] = incl;
+        __syncthreads();
+        if (wid == 0) {
+            int32_t x = lane < kExpandThreads / 32 ? s_wmax[lane] : -1;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int32_t y = __shfl_up_sync(0xffffffffu, x, o);
+                if (lane >= o) x = max(x, y);
+            }
+            if (lane < kExpandThreads / 32) s_wmax[lane] = x;
+        }
+        __syncthreads();
+        const int32_t lane_before = __shfl_up_sync(0xffffffffu, incl, 1);
+        const int32_t before = max(wid > 0 ? s_wmax[wid - 1] : -1, lane > 0 ? lane_before : -1);
+#pragma unroll
+        for (int j = 0; j < kExpandPerThread; j++) sv[tid * kExpandPerThread + j] = max(before, m[j]);
+        __syncthreads();
+        int32_t* out = a.sorted + a.offsets[k];
+        for (int64_t i = tid; i < pend - p0; i += kExpandThreads) out[p0 + i] = sv[i];
     }
+    // the tile's (x', x') pairs, two positions per 16-byte store; NaN past the class's samples
+    float2* pr = a.pairs + a.pair_off[k];
     const float nan = __int_as_float(0x7fc00000);  // quiet NaN pad
     const float off = stage_offset(Lk);              // x + 2^23 is exact for L <= 2^22
-#pragma unroll
-    for (int i = 0; i < kExpandPerThread / 2; i++) {
-        const int idx = (i * 32 + lane) * 2;  // even: the pair store is 16-byte aligned
-        const int64_t q = wbase + idx;
-        if (q < padk) {
-            const float f0 = q < Nk ? (float)wv[(idx >> 3) * 9 + (idx & 7)] + off : nan;
-            const float f1 = q + 1 < Nk ? (float)wv[((idx + 1) >> 3) * 9 + ((idx + 1) & 7)] + off : nan;
-            if (q + 1 < padk) *reinterpret_cast<float4*>(pr + q) = make_float4(f0, f0, f1, f1);
-            else pr[q] = make_float2(f0, f0);
-        }
+    const int64_t qend = min(padk, p0 + kExpandTile);  // padk is a multiple of 128: even
+    for (int64_t i = 2 * (int64_t)tid; p0 + i < qend; i += 2 * kExpandThreads) {
+        const int64_t pos = p0 + i;
+        const float f0 = pos < Nk ? (float)sv[i] + off : nan;
+        const float f1 = pos + 1 < Nk ? (float)sv[i + 1] + off : nan;
+        if (pos + 1 < qend) *reinterpret_cast<float4*>(pr + pos) = make_float4(f0, f0, f1, f1);
+        else pr[pos] = make_float2(f0, f0);
     }
 }
 
@@ -311,6 +340,36 @@ __global__ void k_gather_quantiles(const int32_t* sorted, const int64_t* offsets
 }
 
 }  // namespace
+
+// Histogram blocks of each class (written as a prefix over the classes): slices of at most
+// kHistSlice and at least kHistMinSlice samples, as many as fill whole waves of the device's
+// resident histogram blocks -- a last wave only a little filled would leave most SMs idle.
+cudaError_t hist_block_prefix(const int64_t* N, int32_t K, int32_t* prefix) {
+    int dev = 0, sms = 0, per_sm = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(k_histogram, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 kHistSmemBins * (int)sizeof(int32_t));
+    if (e == cudaSuccess)
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k_histogram, kHistThreads,
+                                                          kHistSmemBins * sizeof(int32_t));
+    if (e != cudaSuccess) return e;
+    const int64_t slots = std::max<int64_t>(1, (int64_t)sms * per_sm);
+    int64_t total = 0, base = 0;
+    for (int32_t k = 0; k < K; k++) {
+        total += N[k];
+        base += (N[k] + kHistSlice - 1) / kHistSlice;
+    }
+    const int64_t target = (base + slots - 1) / slots * slots;
+    const int64_t slice = std::max<int64_t>(kHistMinSlice, (total + target - 1) / target);
+    prefix[0] = 0;
+    for (int32_t k = 0; k < K; k++) {
+        const int64_t nb = std::max<int64_t>((N[k] + kHistSlice - 1) / kHistSlice, N[k] / slice);
+        prefix[k + 1] = (int32_t)std::min<int64_t>(0x7fffffffLL, prefix[k] + std::max<int64_t>(1, nb));
+    }
+    return cudaSuccess;
+}
 
 cudaError_t launch_histogram(const SortArgs& a, int32_t nblocks, cudaStream_t s) {
     // per-device attribute; cheap enough to set on every launch

@@ -281,6 +281,24 @@ def test_the_wait_hook_of_one_context_leaves_another_on_the_same_device_unaffect
         kvdro.kvdro_destroy(plain)
 
 
+@pytest.mark.parametrize("prec", ["exact", "fp32"])
+def test_lam_blocks_keep_the_lowest_index_on_ties_across_a_block_boundary(prec):
+    """More than 128 lam values run as consecutive launches over blocks of 128.  Here the second
+    block repeats the first block's last value (lam = 3) 128 times.  Equal lam values give
+    bit-identical objectives, so a minimum reached at lam = 3 must report index 127 (at eps = 0
+    with c_p = 10 most cells reach it: S does not increase in lam) and no index above 127 may
+    appear; the rest matches the oracle."""
+    rng = np.random.default_rng(17)
+    head = np.logspace(-3, np.log10(3.0), 128)
+    lam = np.concatenate([head, np.full(128, head[-1])])
+    w = make([rng.integers(0, 3000, 5000), rng.integers(0, 3000, 700)], 3000, np.arange(0, 3001, 97), lam,
+             [0.0, 0.5, 20.0, 400.0], [10.0, 0.7], [1.0, 2.0])
+    got = run(w, P[prec])
+    assert got["lam_idx"].max() <= 127
+    assert (got["lam_idx"][0, 0] == 127).any()  # regime c_p = 10, eps = 0
+    compare_full(w, got, O.solve(w), prec)
+
+
 def test_exact_mode_rejects_support_above_its_limit():
     ctx = kvdro.kvdro_create(0)
     try:
