@@ -55,6 +55,9 @@ TERMS_PER_CLK_PER_SM = FMA_TERMS_PER_CLK_PER_SM + ALU_TERMS_PER_CLK_PER_SM
 # The per-term bound of the three-candidate supremum as written: two FMAs, two maxima and one add
 # per term, 5 FP32 lane-operations on 128 FP32 lanes per clock per SM.
 PAPER_FORM_LANE_OPS_PER_TERM = 5.0
+# The FP32-arithmetic kernel's bound: per term one fused multiply-add and one add on the FP32 lanes
+# (2 lane-operations of 128 per clock per SM) and one max on the ALU pipe alongside.
+FP32_PHI_TERMS_PER_CLK_PER_SM = 128.0 / 2.0
 # What the exact kernel evaluates per term: once a cell's exact integer threshold t is known
 # (x >= t exactly when the excess kappa x + d is positive), the excess sum is
 # kappa sum_{x >= t} x + d #{x >= t}, and the kernel streams sum_n |x_n - (t - 1)| to get it.
@@ -80,13 +83,16 @@ def parse_args():
     p.add_argument("--e2e-steps", type=int, default=2)
     p.add_argument("--cpu-seconds", type=float, default=10.0, help="target wall time of the CPU-baseline sample")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-phi-kernel", action="store_true",
+                   help="skip the secondary figure of the per-term phi kernel (roofline.per_term_phi)")
     p.add_argument("--drift-iterations", type=int, default=3)
     p.add_argument("--case", default="",
                    help="WORKLOAD:MODE[:key=val,...], MODE in fp32|fp64|exact|envelope|dual|sort: time one kernel "
                         "path (--warmup untimed, --steps timed runs) and print one line per run.  Keys: L (support "
                         "declared for every class, e.g. 4194305 so FP32 requests take the FP32-arithmetic kernel), "
                         "nl (lam count, log-spaced over the workload's lam range), m (first m regimes), "
-                        "rstride (every rstride-th r)")
+                        "rstride (every rstride-th r), out=all (write every output the contract step writes: "
+                        "cost, lam index, r index, min cost, F-hat; default the r index only)")
     p.add_argument("--suite", action="store_true",
                    help="time every workload in each precision (one JSON line per case) instead of the contract line")
     p.add_argument("--cpu-suite", action="store_true",
@@ -119,6 +125,43 @@ def workload_config(w, world):
         "l2": "flushed between timed steps (256 MiB device write outside the timed events)",
         "parallelism": "single GPU" if world == 1 else f"{world} independent replicas (no data-path collective)",
     }
+
+
+def phi_kernel_figure(kv, w, device, stream, sms, regimes=16, reps=2):
+    """A secondary figure beside the headline: the FP32-arithmetic kernel, which evaluates phi's
+    excess per term (one fused multiply-add, one max and one add per (cell, sample), FP32 sums
+    folded into FP64), on the first `regimes` regimes of the same workload.  The same samples and
+    grid with the support declared as 2^22 + 1, which is what routes FP32 requests to it; the
+    supremum and the sum are unchanged (every sample and reservation lies in both supports)."""
+    import torch
+
+    sub = slice_workload(w, regimes=np.arange(min(regimes, len(w.cp))), name=w.name)
+    L_big = np.full(sub.K, (1 << 22) + 1, np.int32)
+    M, E, K, R, NL = len(sub.cp), len(sub.eps), sub.K, len(sub.r), len(sub.lam)
+    ctx = kv.kvdro_create(device)
+    try:
+        d = torch.from_numpy(sub.samples).to(torch.device("cuda", device))
+        kv.kvdro_load_samples(ctx, K, sub.offsets, d, L_big, sub.L_in, stream)
+        r_idx = torch.empty((M, E, K), dtype=torch.int32, device=d.device)
+        ms = []
+        for i in range(reps + 1):
+            kv.kvdro_eval_grid(ctx, kv.KVDRO_FP32, R, sub.r, NL, sub.lam, E, sub.eps, M, sub.cp, sub.cw,
+                               r_idx=r_idx, stream=stream)
+            if i:
+                ms.append(kv.kvdro_last_grid_ms(ctx))
+    finally:
+        kv.kvdro_destroy(ctx)
+    kernel_ms = statistics.mean(ms)
+    achieved = sub.terms() / (kernel_ms / 1e3)
+    peak_fp32 = sms * FP32_PHI_TERMS_PER_CLK_PER_SM * SM_MAX_MHZ_RECIPE * 1e6
+    peak_paper = sms * 128.0 / PAPER_FORM_LANE_OPS_PER_TERM * SM_MAX_MHZ_RECIPE * 1e6
+    return {"kernel": "k_grid<F32>: per term fma.rn.f32x2 (kappa x + d), max.f32 (excess), add.rn.f32x2 (sum)",
+            "workload": f"{w.name}, first {M} of {len(w.cp)} regimes ({sub.terms():.4g} terms), support declared "
+                        f"as 2^22 + 1", "kernel_ms_mean": kernel_ms, "achieved": achieved, "unit": UNIT,
+            "frac": achieved / peak_fp32,
+            "peak_basis": f"{sms} SMs x {FP32_PHI_TERMS_PER_CLK_PER_SM:.0f} terms/clk/SM (2 FP32 lane-ops per term "
+                          f"on 128 lanes, the max on the ALU pipe) x {SM_MAX_MHZ_RECIPE:.0f} MHz",
+            "frac_survey_basis": achieved / peak_paper}
 
 
 def cpu_model() -> str:
@@ -352,6 +395,8 @@ def run_ours(args):
                 "inst_per_term": inst_per_term}
     if clocks.get("sm_mhz"):
         roofline["frac_at_sampled_clock"] = achieved / (peak * clocks["sm_mhz"] / SM_MAX_MHZ_RECIPE)
+    if not args.no_phi_kernel:
+        roofline["per_term_phi"] = phi_kernel_figure(kv, w, local_rank, stream, sms)
 
     # end to end through the C ABI with host buffers: pinned host samples in, host results out
     h_samples = torch.from_numpy(w.samples).pin_memory()
@@ -546,11 +591,16 @@ def run_cpu_suite(args):
                           "sort_quantiles_s": t_sort, "samples": int(w.N.sum())}), flush=True)
 
 
+def case_options(spec: str) -> dict:
+    parts = spec.split(":")
+    return dict(kv.split("=") for kv in parts[2].split(",")) if len(parts) > 2 and parts[2] else {}
+
+
 def case_workload(spec: str):
     """The workload of a --case spec WORKLOAD:MODE[:key=val,...] and its mode (see --case)."""
     parts = spec.split(":")
     name, mode = parts[0], parts[1]
-    opts = dict(kv.split("=") for kv in parts[2].split(",")) if len(parts) > 2 and parts[2] else {}
+    opts = case_options(spec)
     w = WORKLOADS[name]()
     if "m" in opts or "rstride" in opts:
         regimes = np.arange(int(opts.get("m", len(w.cp))))
@@ -576,13 +626,20 @@ def run_case(args):
     d = torch.from_numpy(w.samples).to(dev)
     r_idx = torch.empty((M, E, K), dtype=torch.int32, device=dev)
     prec = {"fp32": kv.KVDRO_FP32, "fp64": kv.KVDRO_FP64, "exact": kv.KVDRO_EXACT, "envelope": kv.KVDRO_ENVELOPE}
+    outs = {}
+    if case_options(args.case).get("out") == "all" and mode not in ("dual", "sort"):
+        ft = torch.float32 if mode == "fp32" else torch.float64
+        outs = {"cost": torch.empty((M, E, K, R), dtype=ft, device=dev),
+                "lam_idx": torch.empty((M, E, K, R), dtype=torch.int32, device=dev),
+                "min_cost": torch.empty((M, E, K), dtype=ft, device=dev),
+                "fhat": torch.empty((M, E, K), dtype=torch.float64, device=dev)}
     for i in range(args.warmup + args.steps):
         t0 = time.perf_counter()
         kv.kvdro_load_samples(ctx, K, w.offsets, d, w.L, w.L_in)
         if mode == "dual":
             kv.kvdro_eval_dual(ctx, R, w.r, E, w.eps, M, w.cp, w.cw, r_idx=r_idx)
         elif mode != "sort":
-            kv.kvdro_eval_grid(ctx, prec[mode], R, w.r, NL, w.lam, E, w.eps, M, w.cp, w.cw, r_idx=r_idx)
+            kv.kvdro_eval_grid(ctx, prec[mode], R, w.r, NL, w.lam, E, w.eps, M, w.cp, w.cw, r_idx=r_idx, **outs)
         torch.cuda.synchronize(dev)
         line = {"case": args.case, "run": i, "timed": i >= args.warmup, "wall_ms": 1e3 * (time.perf_counter() - t0)}
         if mode not in ("sort", "dual", "envelope"):

@@ -54,16 +54,18 @@ __global__ void __launch_bounds__(kHistThreads) k_histogram(SortArgs a) {
     int32_t* gh = a.hist + a.hist_off[k];
     for (int v = threadIdx.x; v < nb; v += blockDim.x) sh_bins[v] = 0;
     __syncthreads();
+    // Per sample: an unsigned comparison is the whole range check (a negative x wraps above L),
+    // and the two atomics are predicated, so a sample costs no branch.  A thread counts at most
+    // ceil(kHistSlice / kHistThreads) = 128 samples of at most 2^24, so its sum fits 32 bits.
     int bad = 0;
-    unsigned long long sum = 0;
+    uint32_t sum32 = 0;
     auto count = [&](int32_t x) {
-        if (x < 0 || x > Lk) {
-            bad++;
-            return;
-        }
-        sum += (unsigned long long)x;
-        if (x < nb) atomicAdd(&sh_bins[x], 1);
-        else atomicAdd(&gh[x], 1);
+        const bool ok = (uint32_t)x <= (uint32_t)Lk;
+        bad += ok ? 0 : 1;
+        sum32 += ok ? (uint32_t)x : 0u;
+        const bool in_smem = ok && x < nb, in_gmem = ok && x >= nb;
+        if (in_smem) atomicAdd(&sh_bins[x], 1);
+        if (in_gmem) atomicAdd(&gh[x], 1);
     };
     // 16-byte loads of four samples over the slice's aligned middle (alignment is taken from the
     // address: `lengths` is the caller's pointer): each thread loads its next two vectors before
@@ -104,6 +106,7 @@ __global__ void __launch_bounds__(kHistThreads) k_histogram(SortArgs a) {
         const int c = sh_bins[v];
         if (c) atomicAdd(&gh[v], c);
     }
+    unsigned long long sum = sum32;
     for (int o = 16; o; o >>= 1) {
         bad += __shfl_xor_sync(0xffffffffu, bad, o);
         sum += __shfl_xor_sync(0xffffffffu, sum, o);

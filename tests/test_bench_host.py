@@ -116,3 +116,5 @@ def test_case_spec_options():
     w, mode = bench.case_workload("regimes_k8_n2e5:fp32:m=16,nl=256,L=4194305,rstride=4")
     assert mode == "fp32" and len(w.cp) == 16 and len(w.lam) == 256 and len(w.r) == 512
     assert (w.L == 4194305).all() and w.lam[0] == 1e-3 and abs(w.lam[-1] - 1e3) < 1e-9
+    assert bench.case_options("regimes_k8_n2e5:fp32:m=16,out=all") == {"m": "16", "out": "all"}
+    assert bench.case_options("regimes_k8_n2e5:fp32") == {}
