@@ -28,8 +28,9 @@
  *   - Array arguments marked "host or device" may point to either; the library inspects the
  *     pointer.  When any such OUTPUT is in host memory the call blocks until it is filled.
  *     Device outputs are written asynchronously on `stream`.
- *   - The caller owns every buffer it passes; the library owns only what kvdro_create() and
- *     kvdro_load_samples() allocate inside the context, and kvdro_destroy() frees that.
+ *   - The caller owns every buffer it passes; the library owns only what it allocates inside the
+ *     context (the loaded samples' sorted copies and cumulative arrays, and the staging and scratch
+ *     of the evaluation calls, kept for reuse), and kvdro_destroy() frees that.
  *   - A context belongs to one device and one host thread at a time.
  *   - Ties: the minimum over lam and the argmin over r both take the lowest index.
  */
@@ -110,7 +111,11 @@ int kvdro_quantiles(kvdro_ctx* ctx, int32_t F, const double* fractiles, int32_t*
  * KVDRO_FP32 and double for the other modes.
  *   R, r       host int32[R], 1 <= R <= 2^20; every r must satisfy L_in_k <= r <= L_in_k + L_k for
  *              every class (the reservation domain of Sec. 2.2).
- *   NL, lam    host double[NL], finite, >= 0; 1 <= NL <= 256 (128 for KVDRO_FP64).
+ *   NL, lam    host double[NL], finite, >= 0; 1 <= NL <= 256 (128 for KVDRO_FP64).  The exact
+ *              kernel (KVDRO_EXACT, and KVDRO_FP32 when every L_max <= 2^22) takes 128 lam values
+ *              per launch; a larger grid runs as consecutive launches over blocks of 128 with the
+ *              running minimum in context scratch (12 bytes per (regime, eps, class, r), at most
+ *              256 MB at a time).
  *   E, eps     host double[E], finite, >= 0; 1 <= E <= 64.
  *   M, c_p,c_w host double[M] each, finite, >= 0; 1 <= M <= 65536.
  * Outputs (each may be NULL to skip it; host or device):
