@@ -89,6 +89,10 @@ using CfgExact = GridCfg<Prec::EXACT, 2, 8, 0, 2, 512, 4096, 2, 4>;
 // Above a support of 2^19 the packed FP32 sums (exact only up to 2^24) would fold every few loads;
 // there every column takes the integer absolute differences, whose sums fold far less often.
 using CfgExactInt = GridCfg<Prec::EXACT, 2, 8, 0, 2, 512, 4096, 2, 8, 0>;
+// One or two lam values (a small grid, or the last block of a larger one): 8 r x 2 lam tiles, so
+// that a single value pads its tile to 2 columns rather than 8; both columns on the integer sad.
+using CfgExactFewLam = GridCfg<Prec::EXACT, 8, 2, 0, 2, 512, 4096, 2, 8, 0>;
+constexpr int32_t kFewLam = 2;
 constexpr int32_t kExactIntAboveL = 1 << 19;
 constexpr int kWarpsTarget = 16;  // warps per CTA the r groups fill up to
 static_assert(kExactLamBlock == kWarpsTarget * CfgExact::TL && kExactLamBlock == kWarpsTarget * CfgExactInt::TL,
@@ -792,6 +796,7 @@ GridShape grid_shape(Prec p, int32_t R, int32_t NL, int32_t E, int32_t max_L) {
     }
     if (p == Prec::F64) return shape_for<CfgF64>(2, R, NL, E);
     if (p == Prec::EXACT) {  // NL <= kExactLamBlock: larger grids launch in blocks
+        if (NL <= kFewLam) return shape_for<CfgExactFewLam>(8, R, NL, E);
         if (max_L > kExactIntAboveL) return shape_for<CfgExactInt>(6, R, NL, E);
         return shape_for<CfgExact>(3, R, NL, E);
     }
@@ -806,6 +811,8 @@ cudaError_t grid_prepare(Prec p) {
     if (p == Prec::EXACT) {
         cudaError_t e = cudaFuncSetAttribute(k_grid<CfgExact>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
         if (e == cudaSuccess) e = cudaFuncSetAttribute(k_grid<CfgExactInt>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
+        if (e == cudaSuccess)
+            e = cudaFuncSetAttribute(k_grid<CfgExactFewLam>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
         return e;
     }
     if (p == Prec::ENVELOPE)
@@ -825,6 +832,7 @@ cudaError_t launch_grid(Prec p, const GridShape& sh, GridArgs a, cudaStream_t s)
     if (p == Prec::ENVELOPE) k_envelope<<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
     else if (p == Prec::F64) k_grid<CfgF64><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
     else if (p == Prec::EXACT && sh.variant == 3) k_grid<CfgExact><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
+    else if (p == Prec::EXACT && sh.variant == 8) k_grid<CfgExactFewLam><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
     else if (p == Prec::EXACT) k_grid<CfgExactInt><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
     else if (sh.variant == 0) k_grid<CfgF32><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);
     else k_grid<CfgF32Wide><<<(unsigned)nblocks, sh.threads, sh.smem, s>>>(a);

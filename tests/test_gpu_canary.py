@@ -61,7 +61,7 @@ def _check_guards(bufs):
         assert g.guards_intact(), f"{name}: a write outside its extent"
 
 
-CASES = {"narrow": dict(seed=61, n_lam=37), "wide": dict(seed=62, n_lam=200)}
+CASES = {"narrow": dict(seed=61, n_lam=37), "wide": dict(seed=62, n_lam=200), "blocks_of_few": dict(seed=63, n_lam=129)}
 
 
 def _case(kind):
@@ -72,7 +72,8 @@ def _case(kind):
 
 @pytest.mark.parametrize("host", [False, True], ids=["device", "host"])
 @pytest.mark.parametrize("mode,kind", [("fp32", "narrow"), ("fp32", "wide"), ("exact", "narrow"),
-                                       ("exact", "wide"), ("fp64", "narrow"), ("envelope", "narrow")])
+                                       ("exact", "wide"), ("exact", "blocks_of_few"), ("fp64", "narrow"),
+                                       ("envelope", "narrow")])
 def test_grid_outputs_stay_inside_their_extents(mode, kind, host):
     w = _case(kind)
     prec = {"fp32": kvdro.KVDRO_FP32, "fp64": kvdro.KVDRO_FP64, "exact": kvdro.KVDRO_EXACT,
@@ -119,7 +120,7 @@ def test_dual_outputs_stay_inside_their_extents(host):
     check_argmin(bufs["r_idx"].values(), ref["cost"], RTOL["fp64"], "dual r_idx")
 
 
-@pytest.mark.parametrize("kind", ["narrow", "wide"])
+@pytest.mark.parametrize("kind", ["narrow", "wide", "blocks_of_few"])
 def test_noalloc_outputs_stay_inside_their_extents(kind):
     w = _case(kind)
     M, E, K, R, NL = len(w.cp), len(w.eps), w.K, len(w.r), len(w.lam)

@@ -299,6 +299,19 @@ def test_lam_blocks_keep_the_lowest_index_on_ties_across_a_block_boundary(prec):
     compare_full(w, got, O.solve(w), prec)
 
 
+@pytest.mark.parametrize("prec", ["exact", "fp32"])
+@pytest.mark.parametrize("nl,L", [(1, 3000), (2, 3000), (129, 3000), (130, 3000), (1, (1 << 20) + 5), (129, (1 << 20) + 5)])
+def test_one_or_two_lam_values_and_blocks_ending_in_them(prec, nl, L):
+    """A grid of one or two lam values -- or a block of 128 followed by one or two -- takes the
+    8 r x 2 lam tiles (all-integer); a ragged r count (not a multiple of the CTA's 128 rows) and a
+    support above 2^19 included."""
+    rng = np.random.default_rng(nl + L % 97)
+    w = make([np.concatenate([[0, L], rng.integers(0, L + 1, 4100)]), rng.integers(0, L + 1, 333)], L,
+             np.unique(np.linspace(0, L, 203).round()).astype(np.int32), np.logspace(-3, 2, nl),
+             [0.0, 3.0, 250.0], [10.0, 0.4], [1.0, 2.5])
+    compare_full(w, run(w, P[prec]), O.solve(w), prec)
+
+
 def test_exact_mode_rejects_support_above_its_limit():
     ctx = kvdro.kvdro_create(0)
     try:
