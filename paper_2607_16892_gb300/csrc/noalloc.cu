@@ -203,6 +203,20 @@ extern "C" int kvdro_eval_grid_noalloc(int32_t K, const int64_t* offsets, const 
         return report(err, err_len, KVDRO_EINVAL, msg);
     }
 
+    // ---- launch shapes (host only), checked before anything is launched
+    int32_t max_L = 0;
+    for (int32_t k = 0; k < K; k++) max_L = L_max[k] > max_L ? L_max[k] : max_L;
+    const kvdro::Prec kp = exact_ok ? kvdro::Prec::EXACT : kvdro::Prec::F32;
+    const int32_t NL_last = NL - (nblk - 1) * lam_blk;
+    const kvdro::GridShape shape = kvdro::grid_shape(kp, R, NL < lam_blk ? NL : lam_blk, E, max_L);
+    const kvdro::GridShape shape_last = kvdro::grid_shape(kp, R, NL_last, E, max_L);
+    const int64_t per_m = (int64_t)K * (shape.r_blocks > shape_last.r_blocks ? shape.r_blocks : shape_last.r_blocks);
+    // one launch per lam block covers every regime (the running minimum holds all of them), so
+    // with lam blocks the regimes are not split
+    const int64_t m_step = nblk > 1 ? M : (per_m > 0x7fffffffLL ? 1 : 0x7fffffffLL / per_m);
+    if (nblk > 1 && per_m * M > 0x7fffffffLL)
+        return report(err, err_len, KVDRO_EINVAL, "too many CTAs for one launch over every regime");
+
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) {
         cudaGetLastError();
@@ -280,12 +294,6 @@ extern "C" int kvdro_eval_grid_noalloc(int32_t K, const int64_t* offsets, const 
 
     // ---- the grid kernel (the exact one, FP32 outputs, whenever every support is at most 2^22;
     // else the FP32-arithmetic one) and the argmin finalisation
-    int32_t max_L = 0;
-    for (int32_t k = 0; k < K; k++) max_L = L_max[k] > max_L ? L_max[k] : max_L;
-    const kvdro::Prec kp = exact_ok ? kvdro::Prec::EXACT : kvdro::Prec::F32;
-    const int32_t NL_last = NL - (nblk - 1) * lam_blk;
-    const kvdro::GridShape shape = kvdro::grid_shape(kp, R, NL < lam_blk ? NL : lam_blk, E, max_L);
-    const kvdro::GridShape shape_last = kvdro::grid_shape(kp, R, NL_last, E, max_L);
     kvdro::GridArgs a;
     a.pairs = sa.pairs;
     a.pair_off = sa.pair_off;
@@ -325,12 +333,6 @@ extern "C" int kvdro_eval_grid_noalloc(int32_t K, const int64_t* offsets, const 
     a.part_val = nblk > 1 ? reinterpret_cast<double*>(S + o_part_val) : nullptr;
     a.part_idx = nblk > 1 ? reinterpret_cast<int32_t*>(S + o_part_idx) : nullptr;
     const double* d_lam = a.lam;
-    const int64_t per_m = (int64_t)K * (shape.r_blocks > shape_last.r_blocks ? shape.r_blocks : shape_last.r_blocks);
-    // one launch per lam block covers every regime (the running minimum holds all of them), so
-    // with lam blocks the regimes are not split
-    const int64_t m_step = nblk > 1 ? M : (per_m > 0x7fffffffLL ? 1 : 0x7fffffffLL / per_m);
-    if (nblk > 1 && per_m * M > 0x7fffffffLL)
-        return report(err, err_len, KVDRO_EINVAL, "too many CTAs for one launch over every regime");
     for (int64_t m0 = 0; m0 < M; m0 += m_step) {
         a.m0 = (int32_t)m0;
         a.m_count = (int32_t)(m_step < M - m0 ? m_step : M - m0);
