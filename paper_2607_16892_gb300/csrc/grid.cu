@@ -15,7 +15,9 @@
 // Three forms of that sum:
 //  - FP32 and FP64 per term: the excess max(kappa x + d, 0) term by term (one fused multiply-add,
 //    one max, one add per sample and cell) on the base V, or max(-(kappa x + d), 0) on the base
-//    U when nu > mu, whichever cancels less (use_u_split).
+//    U when nu > mu, whichever cancels less (use_u_split).  The excess is evaluated about the
+//    reservation, kappa (x - eta) + W(eta) (excess_at_eta), so that it is exactly zero wherever
+//    it vanishes identically on one side of eta.
 //  - EXACT (also FP32 requests whose supports are all <= 2^22): each cell's integer threshold t
 //    (x >= t exactly when kappa x + d > 0), then per term the exact sum of |x + 1 - t|, half of a
 //    warp's cells on packed FP32 adds and half on integer absolute differences, so the FMA and ALU
@@ -363,8 +365,16 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
     double acc64 = 0.0;  // this lane's cell after the warp transposition
 
     if constexpr (P == Prec::F32) {
-        const float off = stage_offset(a.L[k]);
-        const u64 noff = pk(-off, -off);  // the staged samples carry the class's offset
+        // Each row's excess is taken about its reservation: kappa (x - eta) + W(eta) (excess_at_eta).
+        // x - eta comes from the staged sample in one packed add per row: the staged value carries
+        // the class's offset, and offset + eta is an integer below 2^24, so the add is exact.
+        const double offd = (double)stage_offset(a.L[k]);
+        u64 noff[TR];
+#pragma unroll
+        for (int i = 0; i < TR; i++) {
+            const float o = (float)-(offd + eta[i]);
+            noff[i] = pk(o, o);
+        }
         u64 kap[TL / 2], dd[TR][TL / 2], acc[TR][TL / 2];
 #pragma unroll
         for (int jp = 0; jp < TL / 2; jp++) {
@@ -377,8 +387,8 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
             kap[jp] = pk(v0 ? s0 * (float)(mu0 + nu0) : 0.f, v1 ? s1 * (float)(mu1 + nu1) : 0.f);
 #pragma unroll
             for (int i = 0; i < TR; i++) {
-                const double d0 = excess_offset(cp, cw, mu0, Lk, eta[i]);
-                const double d1 = excess_offset(cp, cw, mu1, Lk, eta[i]);
+                const double d0 = excess_at_eta(cp, cw, mu0, nu0, Lk, eta[i]);
+                const double d1 = excess_at_eta(cp, cw, mu1, nu1, Lk, eta[i]);
                 dd[i][jp] = pk(v0 && rvalid[i] ? s0 * (float)d0 : 0.f, v1 && rvalid[i] ? s1 * (float)d1 : 0.f);
                 acc[i][jp] = 0ull;
             }
@@ -393,11 +403,11 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
 #pragma unroll(C::UNROLL)
                 for (int t = 0; t < nq; t++) {
                     const float4 v = q[lane + 32 * t];  // (x', x') pairs of two samples
-                    const u64 xa = fadd2(pk(v.x, v.y), noff), xb = fadd2(pk(v.z, v.w), noff);
                     // The two samples' excesses are added to each other before they join the running
                     // sum: the same number of adds, half as many additions into the long sum.
 #pragma unroll
-                    for (int i = 0; i < TR; i++)
+                    for (int i = 0; i < TR; i++) {
+                        const u64 xa = fadd2(pk(v.x, v.y), noff[i]), xb = fadd2(pk(v.z, v.w), noff[i]);  // x - eta
 #pragma unroll
                         for (int jp = 0; jp < TL / 2; jp++) {
                             float a0, a1, b0, b1;
@@ -405,6 +415,7 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
                             upk(ffma2(kap[jp], xb, dd[i][jp]), b0, b1);
                             acc[i][jp] = fadd2(acc[i][jp], fadd2(pk(relu(a0), relu(a1)), pk(relu(b0), relu(b1))));
                         }
+                    }
                 }
                 // Every C::FLUSH chunks (and after the last), fold the FP32 partials into the FP64
                 // accumulator of the lane's cell.
@@ -434,7 +445,11 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
             }
         }
     } else if constexpr (P == Prec::F64) {
+        // each row's excess about its reservation, as in the FP32 kernel: x - eta per sample and row
         const double offd = (double)stage_offset(a.L[k]);  // the staged samples carry the class's offset
+        double base[TR];
+#pragma unroll
+        for (int i = 0; i < TR; i++) base[i] = offd + eta[i];  // an exact integer
         double kap[TL], dd[TR][TL], acc[TR][TL];
 #pragma unroll
         for (int j = 0; j < TL; j++) {
@@ -446,7 +461,7 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
             kap[j] = v ? sg * (mu + nu) : 0.0;
 #pragma unroll
             for (int i = 0; i < TR; i++) {
-                dd[i][j] = (v && rvalid[i]) ? sg * excess_offset(cp, cw, mu, Lk, eta[i]) : 0.0;
+                dd[i][j] = (v && rvalid[i]) ? sg * excess_at_eta(cp, cw, mu, nu, Lk, eta[i]) : 0.0;
                 acc[i][j] = 0.0;
             }
         }
@@ -459,14 +474,15 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
                 const int nq = cnt >> 6;
                 for (int t = 0; t < nq; t++) {
                     const float4 v = q[lane + 32 * t];
-                    const double xa = (double)v.x - offd, xb = (double)v.z - offd;  // exact
 #pragma unroll
-                    for (int i = 0; i < TR; i++)
+                    for (int i = 0; i < TR; i++) {
+                        const double xa = (double)v.x - base[i], xb = (double)v.z - base[i];  // x - eta, exact
 #pragma unroll
                         for (int j = 0; j < TL; j++) {
                             acc[i][j] += relu(fma(kap[j], xa, dd[i][j]));
                             acc[i][j] += relu(fma(kap[j], xb, dd[i][j]));
                         }
+                    }
                 }
             }
             consumed = c;

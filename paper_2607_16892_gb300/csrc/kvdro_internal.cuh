@@ -174,6 +174,19 @@ __device__ __forceinline__ double excess_offset(double cp, double cw, double mu,
     return mu == cp ? -__fma_rn(cp, eta, cw_eta) : __dsub_rn(__dmul_rn(cp, L - eta), __fma_rn(mu, L, cw_eta));
 }
 
+// The same excess about the reservation: kappa x + d = kappa (x - eta) + W(eta), with
+//   W(eta) = (c_p - mu)(L - eta) - (c_w - nu) eta,
+// for the per-term kernels, which add max(excess, 0) sample by sample.  x - eta is an exact
+// integer; the two cost differences are exact or rounded once and each product is rounded once,
+// so W(eta) is exactly 0 where the excess vanishes identically on one side of eta -- at the
+// saturated multiplier (mu = c_p, nu = c_w), at eta = L with nu = c_w, at eta = 0 with mu = c_p --
+// and a cell whose every term is zero sums to exactly zero.  (kappa x + d with the rounded d leaves
+// the rounding error of mu L at x = L, which max(., 0) can pass on.)  The differences are at most
+// the costs, so W(eta) is never less accurate than d.
+__device__ __forceinline__ double excess_at_eta(double cp, double cw, double mu, double nu, double L, double eta) {
+    return fma(__dsub_rn(cp, mu), L - eta, -__dmul_rn(__dsub_rn(cw, nu), eta));
+}
+
 // sum_n phi(x_n) with every sample on its own branch: V = c_w eta - nu x for the n - cnt samples
 // below the cell's first active point, U = c_p (L - eta) - mu (L - x) for the cnt samples from it
 // on.  The caller passes exact integer sums: sx_below = sum x below the point, dist_above =

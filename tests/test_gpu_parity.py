@@ -417,3 +417,49 @@ def test_fp32_above_the_exact_limit_matches_the_oracle(nl):
     w = make([rng.integers(0, L + 1, 3000), np.concatenate([[0, L], rng.integers(L - 5000, L + 1, 300)])], L,
              [1, 1 << 21, L - 2, L], np.logspace(-3, 2, nl), [0.0, 1000.0], [10.0, 1.0], [1.0, 1.0])
     compare_full(w, run(w, kvdro.KVDRO_FP32), O.solve(w), "fp32")
+
+
+def _random_shape_case(seed):
+    """A seeded random problem: 1-4 classes of 1-2000 samples (some repeated values), a support
+    from 1 to above 2^22, input lengths, 1-200 reservations, 1-256 lam values, 1-6 radii (eps = 0
+    included), 1-3 regimes with a zero cost now and then."""
+    rng = np.random.default_rng(1000 + seed)
+    K = int(rng.integers(1, 5))
+    L = int(rng.choice([1, 7, 100, 3000, 40000, (1 << 19) + 3], p=[.05, .08, .22, .35, .2, .1]))
+    if seed % 8 == 7:
+        L = (1 << 22) + 9  # FP32 requests take the FP32-arithmetic kernel
+    # input lengths spread by at most L, so that every class shares some reservations
+    L_in = int(rng.integers(0, 50)) + rng.integers(0, min(L, 50) + 1, K) if rng.random() < 0.4 else np.zeros(K, np.int64)
+    cls = []
+    for _ in range(K):
+        n = int(rng.integers(1, 2001))
+        x = rng.integers(0, L + 1, n) if rng.random() < 0.5 else np.minimum(L, rng.geometric(1.0 / max(2, L // 20), n))
+        cls.append(x)
+    lo, hi = int(L_in.max()), int((L_in + L).min())
+    R = int(rng.integers(1, 201))
+    r = np.unique(rng.integers(lo, hi + 1, R))
+    NL = int(rng.integers(1, 257))
+    lam = np.sort(np.concatenate([[0.0] if rng.random() < 0.2 else [], rng.uniform(0, 1, NL) ** 3 * 60]))[:NL]
+    E = int(rng.integers(1, 7))
+    eps = np.concatenate([[0.0], rng.uniform(0, 2 * L + 1, E - 1)])
+    M = int(rng.integers(1, 4))
+    cp = rng.uniform(0, 30, M) * (rng.random(M) > 0.1)
+    cw = rng.uniform(0, 4, M) * (rng.random(M) > 0.1)
+    return make(cls, L, r, lam, eps, cp, cw, L_in=L_in, name=f"sweep{seed}")
+
+
+@pytest.mark.parametrize("seed", range(24))
+def test_random_shapes_every_mode(seed):
+    """Every mode the shape admits (FP32 always; exact up to a support of 2^22; FP64 up to 128 lam
+    values; the envelope mode) against the oracle, on seeded random shapes."""
+    w = _random_shape_case(seed)
+    ref = O.solve(w)
+    modes = ["fp32", "envelope"]
+    if w.L.max() <= (1 << 22):
+        modes.append("exact")
+    if len(w.lam) <= 128:
+        modes.append("fp64")
+    for mode in modes:
+        prec = {"fp32": kvdro.KVDRO_FP32, "fp64": kvdro.KVDRO_FP64, "exact": kvdro.KVDRO_EXACT,
+                "envelope": kvdro.KVDRO_ENVELOPE}[mode]
+        compare_full(w, run(w, prec), ref, "fp32" if mode == "fp32" else "fp64")
