@@ -448,7 +448,7 @@ def _random_shape_case(seed):
     return make(cls, L, r, lam, eps, cp, cw, L_in=L_in, name=f"sweep{seed}")
 
 
-@pytest.mark.parametrize("seed", range(24))
+@pytest.mark.parametrize("seed", range(48))
 def test_random_shapes_every_mode(seed):
     """Every mode the shape admits (FP32 always; exact up to a support of 2^22; FP64 up to 128 lam
     values; the envelope mode) against the oracle, on seeded random shapes."""
@@ -463,3 +463,34 @@ def test_random_shapes_every_mode(seed):
         prec = {"fp32": kvdro.KVDRO_FP32, "fp64": kvdro.KVDRO_FP64, "exact": kvdro.KVDRO_EXACT,
                 "envelope": kvdro.KVDRO_ENVELOPE}[mode]
         compare_full(w, run(w, prec), ref, "fp32" if mode == "fp32" else "fp64")
+
+
+@pytest.mark.parametrize("seed", range(0, 48, 3))
+def test_random_shapes_exact_dual(seed):
+    """The exact dual over gamma >= 0 against the oracle's, on the same seeded random shapes."""
+    from tests.test_gpu_dual import check_dual, run_dual
+    w = _random_shape_case(seed)
+    check_dual(w, run_dual(w), O.solve_dual(w), n_gamma=16, seed=seed)
+
+
+@pytest.mark.parametrize("seed", range(1, 48, 3))
+def test_random_shapes_no_allocation_entry_point(seed):
+    """The allocation-free entry point against the oracle on the same shapes (those whose scratch
+    fits its static array)."""
+    w = _random_shape_case(seed)
+    dev = torch.device("cuda", 0)
+    M, E, K, R, NL = len(w.cp), len(w.eps), w.K, len(w.r), len(w.lam)
+    out = {"cost": torch.empty((M, E, K, R), dtype=torch.float32, device=dev),
+           "lam_idx": torch.empty((M, E, K, R), dtype=torch.int32, device=dev),
+           "r_idx": torch.empty((M, E, K), dtype=torch.int32, device=dev),
+           "min_cost": torch.empty((M, E, K), dtype=torch.float32, device=dev),
+           "fhat": torch.empty((M, E, K), dtype=torch.float64, device=dev)}
+    try:
+        kvdro.kvdro_eval_grid_noalloc(K, w.offsets, torch.from_numpy(w.samples).to(dev), w.L, w.L_in, R, w.r, NL,
+                                      w.lam, E, w.eps, M, w.cp, w.cw, **out)
+    except kvdro.KvdroError as e:
+        if e.status == kvdro.KVDRO_EINVAL and "static scratch" in str(e):
+            pytest.skip("scratch larger than the static array")
+        raise
+    torch.cuda.synchronize()
+    compare_full(w, {k: v.cpu().numpy() for k, v in out.items()}, O.solve(w), "fp32")
