@@ -494,3 +494,44 @@ def test_random_shapes_no_allocation_entry_point(seed):
         raise
     torch.cuda.synchronize()
     compare_full(w, {k: v.cpu().numpy() for k, v in out.items()}, O.solve(w), "fp32")
+
+
+def _random_large_case(seed):
+    """Seeded random shapes with many staged chunks per class (up to 40,000 samples), so that the
+    folds and the chunk ring turn over many times, with ragged last chunks."""
+    rng = np.random.default_rng(5000 + seed)
+    K = int(rng.integers(1, 5))
+    L = int(rng.choice([300, 3000, 40000, 131072, (1 << 19) + 3, (1 << 21) + 1]))
+    if seed % 6 == 5:
+        L = (1 << 22) + 9
+    cls = []
+    for _ in range(K):
+        n = int(rng.integers(1, 40001))
+        cls.append(np.minimum(L, np.rint(np.exp(rng.normal(np.log(max(2.0, rng.uniform(1, L / 4))), 1.0, n)))).astype(np.int64))
+    r = np.unique(rng.integers(0, L + 1, int(rng.integers(1, 301))))
+    NL = int(rng.integers(1, 257))
+    lam = np.sort(rng.uniform(0, 1, NL) ** 3 * 60)
+    E = int(rng.integers(1, 7))
+    eps = np.concatenate([[0.0], rng.uniform(0, 2 * L + 1, E - 1)])
+    M = int(rng.integers(1, 4))
+    cp = rng.uniform(0, 30, M) * (rng.random(M) > 0.1)
+    cw = rng.uniform(0, 4, M) * (rng.random(M) > 0.1)
+    return make(cls, L, r, lam, eps, cp, cw, name=f"large{seed}")
+
+
+@pytest.mark.parametrize("seed", range(18))
+def test_random_large_shapes_every_mode(seed):
+    """Many chunks per class: every cell against the oracle's envelope sums (pinned against the
+    direct sums), and direct per-term sums on sampled cells."""
+    from tests.parity import oracle_from_S
+    w = _random_large_case(seed)
+    S_env = O.envelope_grid(w)
+    ora = oracle_from_S(w, S_env)
+    rng = np.random.default_rng(seed)
+    M, K, R, NL = S_env.shape
+    cells = [rng.integers(0, n, 24) for n in (M, K, R, NL)]
+    direct = O.eval_cells(w, *cells)
+    rel_close(S_env[tuple(cells)], direct, 1e-10, "envelope vs direct")
+    modes = ["fp32"] + (["exact"] if w.L.max() <= (1 << 22) else []) + (["fp64"] if NL <= 128 else [])
+    for mode in modes:
+        compare_full(w, run(w, P[mode]), ora, "fp32" if mode == "fp32" else "fp64")
