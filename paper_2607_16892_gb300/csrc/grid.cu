@@ -608,6 +608,9 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
                 for (int t = t0; t < t1; t++) step(q[lane + 32 * t]);
             }
         };
+        constexpr int kChunkLoads = C::CHUNK / 64;  // loads of one full chunk per lane
+        constexpr int kSegLoads = 32;
+        static_assert(kChunkLoads % kSegLoads == 0, "a full chunk splits into whole segments");
         const int64_t n_k = a.N[k];
         int pending = 0;  // loads since the last fold
         for (int c = 0; c < nchunks; c++) {
@@ -621,15 +624,31 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
                 // which they read as x = 0 (x' = 2^23)
                 const int64_t left = n_k - (int64_t)c * C::CHUNK;
                 const int t_clean = left <= 0 ? 0 : (int)min((int64_t)nq, left >> 6);
-                for (int t0 = 0; t0 < nq; t0 += fe) {
-                    const int t1 = min(nq, t0 + fe);
-                    const int tm = max(t0, min(t1, t_clean));
-                    run(q, t0, tm, false);
-                    if (tm < t1) run(q, tm, t1, true);
-                    pending += t1 - t0;
-                    if (pending >= fe) {
-                        fold();
-                        pending = 0;
+                if (nq == kChunkLoads && t_clean == nq && fe >= kSegLoads) {
+                    // a full chunk of samples only: segments of a fixed trip count, which unroll with
+                    // no remainder.  fe is a power of two >= kSegLoads, so the loads since the last
+                    // fold reach fe exactly at a segment's end.
+#pragma unroll 1
+                    for (int h = 0; h < kChunkLoads / kSegLoads; h++) {
+#pragma unroll(C::UNROLL)
+                        for (int t = 0; t < kSegLoads; t++) step(q[lane + 32 * (kSegLoads * h + t)]);
+                        pending += kSegLoads;
+                        if (pending >= fe) {
+                            fold();
+                            pending = 0;
+                        }
+                    }
+                } else {
+                    for (int t0 = 0; t0 < nq; t0 += fe) {
+                        const int t1 = min(nq, t0 + fe);
+                        const int tm = max(t0, min(t1, t_clean));
+                        run(q, t0, tm, false);
+                        if (tm < t1) run(q, tm, t1, true);
+                        pending += t1 - t0;
+                        if (pending >= fe) {
+                            fold();
+                            pending = 0;
+                        }
                     }
                 }
             }
