@@ -131,8 +131,9 @@ def workload_config(w, world):
 
 def phi_kernel_figure(kv, w, device, stream, sms, regimes=16, reps=2):
     """A secondary figure beside the headline: the FP32-arithmetic kernel, which evaluates phi's
-    excess per term (one fused multiply-add, one max and one add per (cell, sample), FP32 sums
-    folded into FP64), on the first `regimes` regimes of the same workload.  The same samples and
+    excess per term (one saturating fused multiply-add on the excess scaled by a power of two, whose
+    clamp to [0, 1] is the max, and half a packed add per (cell, sample); FP32 sums folded into
+    FP64), on the first `regimes` regimes of the same workload.  The same samples and
     grid with the support declared as 2^22 + 1, which is what routes FP32 requests to it; the
     supremum and the sum are unchanged (every sample and reservation lies in both supports)."""
     import torch
@@ -157,12 +158,13 @@ def phi_kernel_figure(kv, w, device, stream, sms, regimes=16, reps=2):
     achieved = sub.terms() / (kernel_ms / 1e3)
     peak_fp32 = sms * FP32_PHI_TERMS_PER_CLK_PER_SM * SM_MAX_MHZ_RECIPE * 1e6
     peak_paper = sms * 128.0 / PAPER_FORM_LANE_OPS_PER_TERM * SM_MAX_MHZ_RECIPE * 1e6
-    return {"kernel": "k_grid<F32>: per term fma.rn.f32x2 (kappa x + d), max.f32 (excess), add.rn.f32x2 (sum)",
+    return {"kernel": "k_grid<F32>: per term fma.rn.sat.f32 (max(kappa (x - eta) + W, 0) / S, S a power of two), "
+                      "add.rn.f32x2 (sum)",
             "workload": f"{w.name}, first {M} of {len(w.cp)} regimes ({sub.terms():.4g} terms), support declared "
                         f"as 2^22 + 1", "kernel_ms_mean": kernel_ms, "achieved": achieved, "unit": UNIT,
             "frac": achieved / peak_fp32,
             "peak_basis": f"{sms} SMs x {FP32_PHI_TERMS_PER_CLK_PER_SM:.0f} terms/clk/SM (2 FP32 lane-ops per term "
-                          f"on 128 lanes, the max on the ALU pipe) x {SM_MAX_MHZ_RECIPE:.0f} MHz",
+                          f"on 128 lanes: the saturating FMA and the add) x {SM_MAX_MHZ_RECIPE:.0f} MHz",
             "frac_survey_basis": achieved / peak_paper}
 
 

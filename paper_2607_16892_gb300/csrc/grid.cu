@@ -13,11 +13,13 @@
 //   kappa = mu + nu,   d = (c_p - mu) L - (c_p + c_w) eta.
 // Summing over the class: sum_n phi_n = N c_w eta - nu sum_n x_n + sum_n max(kappa x_n + d, 0).
 // Three forms of that sum:
-//  - FP32 and FP64 per term: the excess max(kappa x + d, 0) term by term (one fused multiply-add,
-//    one max, one add per sample and cell) on the base V, or max(-(kappa x + d), 0) on the base
-//    U when nu > mu, whichever cancels less (use_u_split).  The excess is evaluated about the
-//    reservation, kappa (x - eta) + W(eta) (excess_at_eta), so that it is exactly zero wherever
-//    it vanishes identically on one side of eta.
+//  - FP32 and FP64 per term: the excess max(kappa x + d, 0) term by term on the base V, or
+//    max(-(kappa x + d), 0) on the base U when nu > mu, whichever cancels less (use_u_split).  The
+//    excess is evaluated about the reservation, kappa (x - eta) + W(eta) (excess_at_eta), so that
+//    it is exactly zero wherever it vanishes identically on one side of eta.  FP64: one fused
+//    multiply-add, one max and one add per sample and cell.  FP32: one saturating fused
+//    multiply-add on the excess scaled by a power of two (the clamp to [0, 1] is the max) and half
+//    a packed add per sample and cell.
 //  - EXACT (also FP32 requests whose supports are all <= 2^22): each cell's integer threshold t
 //    (x >= t exactly when kappa x + d > 0), then per term the exact sum of |x + 1 - t|, half of a
 //    warp's cells on packed FP32 adds and half on integer absolute differences, so the FMA and ALU
@@ -81,11 +83,11 @@ struct GridCfg {
 // (kExactLamBlock), and the FP32 kernel takes 2 x 16 tiles.  FP64: 2 x 8 tiles.
 // All stage 4096-sample chunks (32 KB) through a 2-deep ring.  The FP32 variants fold their
 // partial sums every 2 chunks (256 samples per lane); the exact variants fold as often as their
-// support size requires.  The narrow FP32 variant unrolls the sample loop 8 times, the exact
-// variants 4 times, and the exact variants give half of every row's lam columns (FCOLS) to the
+// support size requires.  The FP32 and exact variants unroll the sample loop 4 times, and the
+// exact variants give half of every row's lam columns (FCOLS) to the
 // packed FP32 adds, the rest to the integer absolute differences.
-using CfgF32 = GridCfg<Prec::F32, 2, 8, 2, 2, 512, 4096, 2, 8>;
-using CfgF32Wide = GridCfg<Prec::F32, 2, 16, 2, 1, 512, 4096, 2, 2>;
+using CfgF32 = GridCfg<Prec::F32, 2, 8, 2, 2, 512, 4096, 2, 4>;
+using CfgF32Wide = GridCfg<Prec::F32, 2, 16, 2, 1, 512, 4096, 2, 4>;
 using CfgF64 = GridCfg<Prec::F64, 2, 8, 0, 1, 512, 4096, 2>;
 using CfgExact = GridCfg<Prec::EXACT, 2, 8, 0, 2, 512, 4096, 2, 4>;
 // Above a support of 2^19 the packed FP32 sums (exact only up to 2^24) would fold every few loads;
@@ -110,20 +112,16 @@ __device__ __forceinline__ u64 pk(float lo, float hi) {
 __device__ __forceinline__ void upk(u64 r, float& lo, float& hi) {
     asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(r));
 }
-__device__ __forceinline__ u64 ffma2(u64 a, u64 b, u64 c) {
-    u64 r;
-    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
-    return r;
-}
 __device__ __forceinline__ u64 fadd2(u64 a, u64 b) {
     u64 r;
     asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
     return r;
 }
-// max(w, 0); a NaN operand yields 0 (PTX max returns the non-NaN input).
-__device__ __forceinline__ float relu(float w) {
+// a b + c rounded once, then clamped to [0, 1]; a NaN result becomes 0.  For |a b + c| <= 1 this is
+// max(a b + c, 0) in one instruction on the FMA pipe.
+__device__ __forceinline__ float fma_sat(float a, float b, float c) {
     float d;
-    asm("max.f32 %0, %1, 0f00000000;" : "=f"(d) : "f"(w));
+    asm("fma.rn.sat.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
     return d;
 }
 __device__ __forceinline__ u64 abs2(u64 v) {
@@ -131,6 +129,7 @@ __device__ __forceinline__ u64 abs2(u64 v) {
     upk(v, a, b);
     return pk(fabsf(a), fabsf(b));
 }
+// max(w, 0); a NaN operand yields 0 (PTX max returns the non-NaN input).
 __device__ __forceinline__ double relu(double w) {
     double d;
     asm("max.f64 %0, %1, 0d0000000000000000;" : "=d"(d) : "d"(w));
@@ -393,29 +392,72 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
                 acc[i][jp] = 0ull;
             }
         }
+        // One power of two S per warp tile with |kappa (x - eta) + W| <= S for every cell and every
+        // x in [0, L].  The loop sums fma_sat(kappa / S, x - eta, W / S) = max(excess, 0) / S, and the
+        // fold multiplies the reduced sums by S.  Scaling by a power of two changes no rounding, so
+        // the sums equal those of a separate max per term, with the max folded into the FMA.
+        double wmax = 1.0;
+#pragma unroll
+        for (int jp = 0; jp < TL / 2; jp++) {
+            float k0, k1;
+            upk(kap[jp], k0, k1);
+#pragma unroll
+            for (int i = 0; i < TR; i++) {
+                float d0, d1;
+                upk(dd[i][jp], d0, d1);
+                const double xm = fmax(fabs(eta[i]), fabs(Lk - eta[i]));  // largest |x - eta|
+                wmax = fmax(wmax, fmax(fabs((double)k0) * xm + fabs((double)d0), fabs((double)k1) * xm + fabs((double)d1)));
+            }
+        }
+        int sexp;
+        (void)frexp(wmax, &sexp);  // wmax < 2^sexp
+        const float S = ldexpf(1.f, sexp), invS = ldexpf(1.f, -sexp);
+#pragma unroll
+        for (int jp = 0; jp < TL / 2; jp++) {
+            float k0, k1;
+            upk(kap[jp], k0, k1);
+            kap[jp] = pk(k0 * invS, k1 * invS);
+#pragma unroll
+            for (int i = 0; i < TR; i++) {
+                float d0, d1;
+                upk(dd[i][jp], d0, d1);
+                dd[i][jp] = pk(d0 * invS, d1 * invS);
+            }
+        }
+        // one load: two samples' excesses for every cell of the tile.  The two samples' excesses are
+        // added to each other before they join the running sum: the same number of adds, half as
+        // many additions into the long sum.
+        auto step = [&](const float4 v) {
+#pragma unroll
+            for (int i = 0; i < TR; i++) {
+                const u64 xa = fadd2(pk(v.x, v.y), noff[i]), xb = fadd2(pk(v.z, v.w), noff[i]);  // x - eta
+                float xa0, xa1, xb0, xb1;
+                upk(xa, xa0, xa1);
+                upk(xb, xb0, xb1);
+#pragma unroll
+                for (int jp = 0; jp < TL / 2; jp++) {
+                    float k0, k1, d0, d1;
+                    upk(kap[jp], k0, k1);
+                    upk(dd[i][jp], d0, d1);
+                    const float a0 = fma_sat(k0, xa0, d0), a1 = fma_sat(k1, xa0, d1);
+                    const float b0 = fma_sat(k0, xb0, d0), b1 = fma_sat(k1, xb0, d1);
+                    acc[i][jp] = fadd2(acc[i][jp], fadd2(pk(a0, a1), pk(b0, b1)));
+                }
+            }
+        };
         for (int c = 0; c < nchunks; c++) {
             const int s = c % C::STAGES;
             if (!mbar_wait_bounded(smem_u32(&full[s]), (uint32_t)((c / C::STAGES) & 1), a.wait_ns)) timeout = true;
             if (!timeout) {
                 const int cnt = (int)min((int64_t)C::CHUNK, np - (int64_t)c * C::CHUNK);
                 const float4* q = reinterpret_cast<const float4*>(ring + (size_t)s * C::CHUNK);
-                const int nq = cnt >> 6;  // float4 (two samples) per lane
+                const int nq = cnt >> 6;  // float4 (two samples) per lane: (x', x') pairs
+                if (nq == C::CHUNK / 64) {  // a full chunk: a fixed trip count, unrolled with no remainder
 #pragma unroll(C::UNROLL)
-                for (int t = 0; t < nq; t++) {
-                    const float4 v = q[lane + 32 * t];  // (x', x') pairs of two samples
-                    // The two samples' excesses are added to each other before they join the running
-                    // sum: the same number of adds, half as many additions into the long sum.
-#pragma unroll
-                    for (int i = 0; i < TR; i++) {
-                        const u64 xa = fadd2(pk(v.x, v.y), noff[i]), xb = fadd2(pk(v.z, v.w), noff[i]);  // x - eta
-#pragma unroll
-                        for (int jp = 0; jp < TL / 2; jp++) {
-                            float a0, a1, b0, b1;
-                            upk(ffma2(kap[jp], xa, dd[i][jp]), a0, a1);
-                            upk(ffma2(kap[jp], xb, dd[i][jp]), b0, b1);
-                            acc[i][jp] = fadd2(acc[i][jp], fadd2(pk(relu(a0), relu(a1)), pk(relu(b0), relu(b1))));
-                        }
-                    }
+                    for (int t = 0; t < C::CHUNK / 64; t++) step(q[lane + 32 * t]);
+                } else {
+#pragma unroll 1
+                    for (int t = 0; t < nq; t++) step(q[lane + 32 * t]);
                 }
                 // Every C::FLUSH chunks (and after the last), fold the FP32 partials into the FP64
                 // accumulator of the lane's cell.
@@ -428,7 +470,7 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
                             upk(acc[i][jp], vals[i * TL + 2 * jp], vals[i * TL + 2 * jp + 1]);
                             acc[i][jp] = 0ull;
                         }
-                    acc64 += (double)transpose_reduce<float, V>(vals, lane);
+                    acc64 += (double)transpose_reduce<float, V>(vals, lane) * (double)S;
                 }
             }
             consumed = c;
