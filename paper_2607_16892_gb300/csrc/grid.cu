@@ -365,8 +365,9 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
 
     if constexpr (P == Prec::F32) {
         // Each row's excess is taken about its reservation: kappa (x - eta) + W(eta) (excess_at_eta).
-        // x - eta comes from the staged sample in one packed add per row: the staged value carries
-        // the class's offset, and offset + eta is an integer below 2^24, so the add is exact.
+        // x - eta comes from the staged samples in one packed add per row and load (both samples of
+        // the load): the staged value carries the class's offset, and offset + eta is an integer
+        // below 2^24, so the add is exact.
         const double offd = (double)stage_offset(a.L[k]);
         u64 noff[TR];
 #pragma unroll
@@ -430,10 +431,10 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
         auto step = [&](const float4 v) {
 #pragma unroll
             for (int i = 0; i < TR; i++) {
-                const u64 xa = fadd2(pk(v.x, v.y), noff[i]), xb = fadd2(pk(v.z, v.w), noff[i]);  // x - eta
-                float xa0, xa1, xb0, xb1;
-                upk(xa, xa0, xa1);
-                upk(xb, xb0, xb1);
+                // x - eta of the load's two samples in one packed add (v.x and v.z: one copy of each)
+                const u64 xab = fadd2(pk(v.x, v.z), noff[i]);
+                float xa0, xb0;
+                upk(xab, xa0, xb0);
 #pragma unroll
                 for (int jp = 0; jp < TL / 2; jp++) {
                     float k0, k1, d0, d1;
@@ -781,6 +782,48 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
 constexpr int kEnvR = 8;          // r values per CTA
 constexpr int kEnvThreads = 256;
 
+// Order key of a double for the minimum over lam: equal for equal values (-0 is taken as +0) and
+// ordered as the values are for every non-NaN double, so the comparison runs on integers instead
+// of the FP64 pipe (which this part executes at 2 operations per clock per SM).
+__device__ __forceinline__ long long order_key(double v) {
+    long long b = __double_as_longlong(v);
+    if (b == (long long)0x8000000000000000ull) b = 0;
+    return b ^ ((b >> 63) & 0x7fffffffffffffffll);
+}
+
+// The envelope kernel's epilogue: each thread takes whole (r, eps) pairs and scans lam in
+// ascending order with a strict comparison, so ties keep the lowest index (as cta_epilogue's
+// reduction does); the cost of every lam is lam * eps + S, rounded as there.  One FP64 multiply
+// and one add per (r, eps, lam), no shuffles.
+__device__ __forceinline__ void env_epilogue(const GridArgs& a, const double* s_S, const double* s_lam,
+                                             const double* s_eps, int r_cta0, int m, int k) {
+    for (int p = threadIdx.x; p < kEnvR * a.E; p += blockDim.x) {
+        const int rl = p / a.E, e = p % a.E;
+        const int ri = r_cta0 + rl;
+        if (ri >= a.R) continue;
+        const double eps = s_eps[e];
+        const double* S = s_S + rl * a.NL;
+        double best = __dadd_rn(__dmul_rn(s_lam[0], eps), S[0]);
+        long long best_key = order_key(best);
+        int bj = 0;
+        for (int j = 1; j < a.NL; j++) {
+            const double v = __dadd_rn(__dmul_rn(s_lam[j], eps), S[j]);
+            const long long key = order_key(v);
+            if (key < best_key) {
+                best_key = key;
+                best = v;
+                bj = j;
+            }
+        }
+        const size_t row = ((size_t)m * a.E + e) * a.K + k;
+        const size_t o = row * a.R + ri;
+        static_cast<double*>(a.cost_out)[o] = best;
+        if (a.lam_idx_out) a.lam_idx_out[o] = bj + a.lam0;
+        const u64 key = ((u64)__double_as_longlong(best > 0.0 ? best : 0.0) & ~0xFFFFFull) | (u64)ri;
+        atomicMin(a.keys + row, key);
+    }
+}
+
 __global__ void __launch_bounds__(kEnvThreads) k_envelope(const GridArgs a) {
     extern __shared__ __align__(16) double esm[];
     double* s_lam = esm;
@@ -819,7 +862,7 @@ __global__ void __launch_bounds__(kEnvThreads) k_envelope(const GridArgs a) {
         if (a.S_out) static_cast<double*>(a.S_out)[(((size_t)m * a.K + k) * a.R + ri) * a.NL_out + a.lam0 + j] = S;
     }
     __syncthreads();
-    cta_epilogue<false>(a, s_S, s_lam, s_eps, a.NL, kEnvR, r_cta0, m, k);
+    env_epilogue(a, s_S, s_lam, s_eps, r_cta0, m, k);
 }
 
 template <Prec P>
