@@ -81,21 +81,22 @@ struct GridCfg {
 // 2 r x 8 lam tiles, up to 16 warps per CTA and (FP32, exact) two CTAs per SM (64 registers)
 // for up to 128 lam values; larger lam grids run the exact kernel in blocks of 128 lam values
 // (kExactLamBlock), and the FP32 kernel takes 2 x 16 tiles.  FP64: 2 x 8 tiles.
-// All stage 4096-sample chunks (32 KB) through a 2-deep ring.  The FP32 variants fold their
-// partial sums every 2 chunks (256 samples per lane); the exact variants fold as often as their
-// support size requires.  The FP32 and exact variants unroll the sample loop 4 times, and the
-// exact variants give half of every row's lam columns (FCOLS) to the
-// packed FP32 adds, the rest to the integer absolute differences.
+// The exact variants stage 6144-sample chunks (48 KB), the FP32 and FP64 ones 4096-sample chunks
+// (32 KB), through a 2-deep ring (two CTAs of the exact kernel per SM: 2 x 96 KB of ring).  The FP32
+// variants fold their partial sums every 2 chunks (256 samples per lane); the exact variants fold
+// as often as their support size requires, independently of the chunk size.  The FP32 and exact
+// variants unroll the sample loop 4 times, and the exact variants give half of every row's lam
+// columns (FCOLS) to the packed FP32 adds, the rest to the integer absolute differences.
 using CfgF32 = GridCfg<Prec::F32, 2, 8, 2, 2, 512, 4096, 2, 4>;
 using CfgF32Wide = GridCfg<Prec::F32, 2, 16, 2, 1, 512, 4096, 2, 4>;
 using CfgF64 = GridCfg<Prec::F64, 2, 8, 0, 1, 512, 4096, 2>;
-using CfgExact = GridCfg<Prec::EXACT, 2, 8, 0, 2, 512, 4096, 2, 4>;
+using CfgExact = GridCfg<Prec::EXACT, 2, 8, 0, 2, 512, 6144, 2, 4>;
 // Above a support of 2^19 the packed FP32 sums (exact only up to 2^24) would fold every few loads;
 // there every column takes the integer absolute differences, whose sums fold far less often.
-using CfgExactInt = GridCfg<Prec::EXACT, 2, 8, 0, 2, 512, 4096, 2, 8, 0>;
+using CfgExactInt = GridCfg<Prec::EXACT, 2, 8, 0, 2, 512, 6144, 2, 8, 0>;
 // One or two lam values (a small grid, or the last block of a larger one): 8 r x 2 lam tiles, so
 // that a single value pads its tile to 2 columns rather than 8; both columns on the integer sad.
-using CfgExactFewLam = GridCfg<Prec::EXACT, 8, 2, 0, 2, 512, 4096, 2, 8, 0>;
+using CfgExactFewLam = GridCfg<Prec::EXACT, 8, 2, 0, 2, 512, 6144, 2, 8, 0>;
 constexpr int32_t kFewLam = 2;
 constexpr int32_t kExactIntAboveL = 1 << 19;
 constexpr int kWarpsTarget = 16;  // warps per CTA the r groups fill up to
@@ -669,8 +670,10 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
                 const int t_clean = left <= 0 ? 0 : (int)min((int64_t)nq, left >> 6);
                 if (nq == kChunkLoads && t_clean == nq && fe >= kSegLoads) {
                     // a full chunk of samples only: segments of a fixed trip count, which unroll with
-                    // no remainder.  fe is a power of two >= kSegLoads, so the loads since the last
-                    // fold reach fe exactly at a segment's end.
+                    // no remainder.  fe is a power of two >= kSegLoads and every earlier chunk took
+                    // this path too (only a class's last chunk is ragged or padded), so the loads
+                    // since the last fold are a multiple of kSegLoads and reach fe exactly at a
+                    // segment's end.
 #pragma unroll 1
                     for (int h = 0; h < kChunkLoads / kSegLoads; h++) {
 #pragma unroll(C::UNROLL)
@@ -685,6 +688,10 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
                     for (int t0 = 0; t0 < nq; t0 += fe) {
                         const int t1 = min(nq, t0 + fe);
                         const int tm = max(t0, min(t1, t_clean));
+                        if (pending + (t1 - t0) > fe) {  // fold first: the loads since the last fold would pass fe
+                            fold();
+                            pending = 0;
+                        }
                         run(q, t0, tm, false);
                         if (tm < t1) run(q, tm, t1, true);
                         pending += t1 - t0;

@@ -223,7 +223,7 @@ def test_a_wait_that_runs_out_reports_etimeout_and_the_device_stays_usable(monke
     drains the copies it did issue and sets the error bit, and the call reports KVDRO_ETIMEOUT.
     Afterwards the same CUDA context evaluates correctly."""
     rng = np.random.default_rng(3)
-    w = make([rng.integers(0, 900, 20000)], 1000, [10, 200, 600], [0.5, 5.0], [0.0, 10.0], 10.0, 1.0)  # 5 chunks
+    w = make([rng.integers(0, 900, 20000)], 1000, [10, 200, 600], [0.5, 5.0], [0.0, 10.0], 10.0, 1.0)  # 4 staged chunks in the exact kernel, 5 in the FP64 one
     monkeypatch.setenv("KVDRO_TEST_SKIP_CHUNK", "2")
     ctx = kvdro.kvdro_create(0)
     monkeypatch.delenv("KVDRO_TEST_SKIP_CHUNK")
@@ -535,3 +535,24 @@ def test_random_large_shapes_every_mode(seed):
     modes = ["fp32"] + (["exact"] if w.L.max() <= (1 << 22) else []) + (["fp64"] if NL <= 128 else [])
     for mode in modes:
         compare_full(w, run(w, P[mode]), ora, "fp32" if mode == "fp32" else "fp64")
+
+
+@pytest.mark.parametrize("L", [65534, 32767, 16382, 131070])
+def test_exact_sums_stay_exact_at_the_fold_bound(L):
+    """The exact kernel folds its packed FP32 sums after fe loads, fe the largest power of two with
+    2 fe (L + 1) <= 2^24; each L here sits just below such a bound, so a lane's sums reach nearly
+    2^24 by the fold.  Samples crowd the top of the support and the reservations its bottom (every
+    |x - c| near L, odd and even), and the classes end in a large ragged chunk after one, two or
+    three full ones, so the loads since the last fold do not restart at a chunk boundary.  One load
+    past the bound rounds the sums: the exact mode must still meet the envelope mode (same integer
+    sums, O(1) per cell) to 1e-12 and the oracle to 1e-9."""
+    rng = np.random.default_rng(L)
+    sizes = (12144, 3 * 6144 + 6100, 2 * 6144 + 6100, 4 * 4096 + 4000)
+    cls = [L - rng.integers(0, 1 + L // 64, n) for n in sizes]
+    r = np.array([0, 1, 2, 3, 7, 30, L // 2, L - 1, L])
+    lam = np.array([0.01, 0.7, 1.0, 3.0, 9.5, 10.0, 25.0, 1e3])  # below, at and above c_w and c_p
+    w = make(cls, L, r, lam, [0.0, 5.0, 300.0], [10.0, 1.0], [1.0, 2.0], name=f"foldbound{L}")
+    ex, env = run(w, kvdro.KVDRO_EXACT), run(w, kvdro.KVDRO_ENVELOPE)
+    np.testing.assert_allclose(ex["S"], env["S"], rtol=1e-12, atol=0)
+    compare_full(w, ex, O.solve(w), "exact")
+    compare_full(w, run(w, P["fp32"]), O.solve(w), "fp32")

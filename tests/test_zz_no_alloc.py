@@ -120,7 +120,7 @@ def test_noalloc_reports_a_wait_that_runs_out(monkeypatch):
     never issued; the call returns KVDRO_ETIMEOUT (its outputs are incomplete) instead of
     KVDRO_OK, and the next call without the hook is correct."""
     rng = np.random.default_rng(5)
-    cls = rng.integers(0, 900, 20000).astype(np.int32)  # five staged chunks
+    cls = rng.integers(0, 900, 20000).astype(np.int32)  # four staged chunks
     w = Workload(name="wait", samples=cls, offsets=np.array([0, cls.size], np.int64), L=np.array([1000], np.int32),
                  L_in=np.zeros(1, np.int32), r=np.array([10, 200, 600], np.int32), lam=np.array([0.5, 5.0]),
                  eps=np.array([0.0, 10.0]), cp=np.array([10.0]), cw=np.array([1.0]), fractiles=np.array([0.5]))
