@@ -38,6 +38,9 @@ constexpr long long kTestWaitNs = 1000000;  // the wait test's bound: 1 ms
 constexpr int32_t kMaxNLf32 = 256;
 constexpr int64_t kPartBytes = 256LL << 20;  // cap of the running-minimum buffer of lam blocks
 constexpr int32_t kMaxNLf64 = 128;
+// Host outputs of a grid over several regimes return in up to this many regime blocks, each
+// copied while the next evaluates.
+constexpr int64_t kCopyBlocks = 16;
 
 struct Buf {
     void* p = nullptr;
@@ -66,6 +69,9 @@ struct kvdro_ctx {
     size_t pin_bytes = 0;
     cudaEvent_t pin_free = nullptr;  // completes when the last copy out of `pin` is done
     cudaEvent_t grid_t0 = nullptr, grid_t1 = nullptr;  // around the last grid-kernel launches
+    // Copies of host outputs back to the caller, overlapped with later grid launches
+    cudaStream_t copy_stream = nullptr;
+    cudaEvent_t copy_ready = nullptr, copy_done = nullptr;
     bool grid_timed = false;
 
     // device views into `meta`
@@ -240,7 +246,10 @@ int kvdro_create(kvdro_ctx** out, int device_ordinal) {
         cudaEventCreateWithFlags(&ctx->pin_free, cudaEventDisableTiming) != cudaSuccess ||
         kvdro::grid_prepare(Prec::EXACT) != cudaSuccess || kvdro::grid_prepare(Prec::ENVELOPE) != cudaSuccess ||
         cudaEventCreate(&ctx->grid_t0) != cudaSuccess ||
-        cudaEventCreate(&ctx->grid_t1) != cudaSuccess) {
+        cudaEventCreate(&ctx->grid_t1) != cudaSuccess ||
+        cudaStreamCreateWithFlags(&ctx->copy_stream, cudaStreamNonBlocking) != cudaSuccess ||
+        cudaEventCreateWithFlags(&ctx->copy_ready, cudaEventDisableTiming) != cudaSuccess ||
+        cudaEventCreateWithFlags(&ctx->copy_done, cudaEventDisableTiming) != cudaSuccess) {
         cudaGetLastError();
         delete ctx;
         return KVDRO_ECUDA;
@@ -261,6 +270,9 @@ int kvdro_destroy(kvdro_ctx* ctx) {
     if (ctx->pin_free) cudaEventDestroy(ctx->pin_free);
     if (ctx->grid_t0) cudaEventDestroy(ctx->grid_t0);
     if (ctx->grid_t1) cudaEventDestroy(ctx->grid_t1);
+    if (ctx->copy_ready) cudaEventDestroy(ctx->copy_ready);
+    if (ctx->copy_done) cudaEventDestroy(ctx->copy_done);
+    if (ctx->copy_stream) cudaStreamDestroy(ctx->copy_stream);
     cudaGetLastError();
     delete ctx;
     return KVDRO_OK;
@@ -605,6 +617,12 @@ int kvdro_eval_grid(kvdro_ctx* ctx, int precision, int32_t R, const int32_t* r, 
         a.part_val = static_cast<double*>(ctx->part.p);
         a.part_idx = reinterpret_cast<int32_t*>(static_cast<char*>(ctx->part.p) + (size_t)cells * 8);
     }
+    // Host outputs laid out regime-major (S, cost, lam index) go back in blocks of regimes on the
+    // context's copy stream, each block as soon as its launches are done, so the copies overlap the
+    // evaluation of later regimes instead of following the whole grid.
+    const bool pipe = M > 1 && ((outs[0].user && outs[0].host) || (outs[1].user && outs[1].host) ||
+                                (outs[2].user && outs[2].host));
+    if (pipe) m_step = std::min<int64_t>(m_step, (M + kCopyBlocks - 1) / kCopyBlocks);
     ctx->grid_timed = false;
     KV_CUDA(cudaEventRecord(ctx->grid_t0, s), "recording grid start");
     for (int64_t m0 = 0; m0 < M; m0 += m_step) {
@@ -617,6 +635,19 @@ int kvdro_eval_grid(kvdro_ctx* ctx, int precision, int32_t R, const int32_t* r, 
             a.part_first = b == 0;
             a.part_last = b + 1 == nblk;
             KV_CUDA(kvdro::launch_grid(KP, b + 1 < nblk ? shape : shape_last, a, s), "grid kernel");
+        }
+        if (pipe) {
+            KV_CUDA(cudaEventRecord(ctx->copy_ready, s), "recording a regime block");
+            KV_CUDA(cudaStreamWaitEvent(ctx->copy_stream, ctx->copy_ready, 0), "ordering a copy");
+            for (int i = 0; i < 3; i++) {
+                const Out& x = outs[i];
+                if (!x.user || !x.host) continue;
+                const size_t per_m = x.bytes / (size_t)M;
+                KV_CUDA(cudaMemcpyAsync(static_cast<char*>(x.user) + (size_t)m0 * per_m,
+                                        static_cast<const char*>(x.dev) + (size_t)m0 * per_m,
+                                        (size_t)a.m_count * per_m, cudaMemcpyDeviceToHost, ctx->copy_stream),
+                        "copying results");
+            }
         }
     }
     KV_CUDA(cudaEventRecord(ctx->grid_t1, s), "recording grid end");
@@ -640,9 +671,15 @@ int kvdro_eval_grid(kvdro_ctx* ctx, int precision, int32_t R, const int32_t* r, 
     if (fa.r_idx || fa.min_cost || fa.fhat) KV_CUDA(kvdro::launch_finalize(P, fa, s), "finalize kernel");
 
     if (stage_bytes) {
-        for (Out& x : outs)
-            if (x.user && x.host)
+        if (pipe) {  // the regime blocks' copies, then the rest on the caller's stream
+            KV_CUDA(cudaEventRecord(ctx->copy_done, ctx->copy_stream), "recording the copies");
+            KV_CUDA(cudaStreamWaitEvent(s, ctx->copy_done, 0), "ordering the copies");
+        }
+        for (int i = 0; i < 6; i++) {
+            const Out& x = outs[i];
+            if (x.user && x.host && !(pipe && i < 3))
                 KV_CUDA(cudaMemcpyAsync(x.user, x.dev, x.bytes, cudaMemcpyDeviceToHost, s), "copying results");
+        }
         KV_CUDA(cudaStreamSynchronize(s), "copying results");
         return check_kernel_errors(ctx, s);
     }

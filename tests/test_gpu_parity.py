@@ -113,6 +113,20 @@ def test_host_buffers_match_device_buffers(prec):
         assert np.array_equal(a[k], b[k]), k
 
 
+@pytest.mark.parametrize("prec", ["fp64", "fp32", "exact", "envelope"])
+def test_host_outputs_copied_in_regime_blocks_match_device_outputs(prec):
+    """With many regimes, host outputs come back in blocks of regimes on the context's copy
+    stream while later blocks evaluate: 37 regimes make blocks of 3 with a ragged last one, and
+    150 lam values (100 in FP64) make the exact kernel run two lam blocks per regime block."""
+    w = random_case(23, K=2, N=(2500, 90), L=(900, 900), R=13, n_lam=100 if prec == "fp64" else 150, n_eps=3, M=37,
+                    lam_range=(1e-3, 50.0), eps_max=200.0)
+    mode = kvdro.KVDRO_ENVELOPE if prec == "envelope" else P[prec]
+    a = run(w, mode)
+    b = run(w, mode, host_outputs=True)
+    for k in a:
+        assert np.array_equal(a[k], b[k]), k
+
+
 def test_repeatable_bit_for_bit():
     w = random_case(22, K=2, N=(9000, 300), L=(2000, 2000), R=40, n_lam=50, n_eps=3, M=2)
     a = run(w, kvdro.KVDRO_FP32)
