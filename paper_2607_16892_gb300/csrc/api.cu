@@ -623,6 +623,14 @@ int kvdro_eval_grid(kvdro_ctx* ctx, int precision, int32_t R, const int32_t* r, 
     const bool pipe = M > 1 && ((outs[0].user && outs[0].host) || (outs[1].user && outs[1].host) ||
                                 (outs[2].user && outs[2].host));
     if (pipe) m_step = std::min<int64_t>(m_step, (M + kCopyBlocks - 1) / kCopyBlocks);
+    // Whatever way the call returns, no copy into the caller's host buffers is still in flight.
+    struct CopyDrain {
+        cudaStream_t cs;
+        bool armed;
+        ~CopyDrain() {
+            if (armed) cudaStreamSynchronize(cs);
+        }
+    } drain{ctx->copy_stream, pipe};
     ctx->grid_timed = false;
     KV_CUDA(cudaEventRecord(ctx->grid_t0, s), "recording grid start");
     for (int64_t m0 = 0; m0 < M; m0 += m_step) {
