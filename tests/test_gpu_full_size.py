@@ -47,12 +47,40 @@ def direct_cells(w, gpu_S, n, rtol, seed):
     return rel_close(gpu_S[m, k, r, l], ref, rtol, "S (direct cells)")
 
 
+def chosen_r_cells(w, gpu_S, gpu_r_idx, rtol, seed, max_terms=4e9):
+    """The direct per-term oracle at every cell of each (regime, class)'s chosen reservations and
+    their neighbours: r* and r* +- 1 over every radius, every lam value -- or, when that would pass
+    max_terms terms, a seeded subset of the lam values that keeps each row's chosen ones."""
+    rng = np.random.default_rng(seed)
+    M, K, R, NL = gpu_S.shape
+    cells = []
+    for mm in range(M):
+        for k in range(K):
+            rs = np.unique(np.clip(np.concatenate([gpu_r_idx[mm, :, k] + d for d in (-1, 0, 1)]), 0, R - 1))
+            for ri in rs:
+                cells.append((mm, k, ri))
+    cells = np.array(cells, np.int64)
+    n_per = int(np.mean(w.N))
+    keep = NL if len(cells) * NL * n_per <= max_terms else max(4, int(max_terms // (len(cells) * n_per)))
+    m, k, r, l = [], [], [], []
+    for mm, kk, ri in cells:
+        lams = np.arange(NL) if keep >= NL else rng.choice(NL, keep, replace=False)
+        m.append(np.full(len(lams), mm))
+        k.append(np.full(len(lams), kk))
+        r.append(np.full(len(lams), ri))
+        l.append(lams)
+    m, k, r, l = (np.concatenate(v) for v in (m, k, r, l))
+    ref = O.eval_cells(w, m, k, r, l)
+    return rel_close(gpu_S[m, k, r, l], ref, rtol, "S (cells at the chosen r)")
+
+
 def test_lognormal_k8_n1e5_fp32_full_grid_as_benchmarked():
     w = lognormal_workload_k8_n1e5()
     gpu = run(w, kvdro.KVDRO_FP32)
     S_env = O.envelope_grid(w)
     rep = compare_full(w, gpu, oracle_from_S(w, S_env), "fp32")
-    rep["direct"] = direct_cells(w, gpu["S"], 2048, RTOL["fp32"], 1)
+    rep["direct"] = direct_cells(w, gpu["S"], 4096, RTOL["fp32"], 1)
+    rep["direct_at_r_star"] = chosen_r_cells(w, gpu["S"], gpu["r_idx"], RTOL["fp32"], 11)
     assert rep["r_idx_exact"] > 0
     print(rep)
 
@@ -62,7 +90,8 @@ def test_lognormal_k8_n1e5_exact_full_grid():
     w = lognormal_workload_k8_n1e5()
     gpu = run(w, kvdro.KVDRO_EXACT)
     rep = compare_full(w, gpu, oracle_from_S(w, O.envelope_grid(w)), "exact")
-    rep["direct"] = direct_cells(w, gpu["S"], 1024, RTOL["exact"], 7)
+    rep["direct"] = direct_cells(w, gpu["S"], 4096, RTOL["exact"], 7)
+    rep["direct_at_r_star"] = chosen_r_cells(w, gpu["S"], gpu["r_idx"], RTOL["exact"], 17)
     print(rep)
 
 
@@ -70,7 +99,8 @@ def test_heavy_tail_k16_n1e6_exact_full_grid():
     w = heavy_tail_workload_k16_n1e6()
     gpu = run(w, kvdro.KVDRO_EXACT)
     rep = compare_full(w, gpu, oracle_from_S(w, O.envelope_grid(w)), "exact")
-    rep["direct"] = direct_cells(w, gpu["S"], 128, RTOL["exact"], 8)
+    rep["direct"] = direct_cells(w, gpu["S"], 4096, RTOL["exact"], 8)
+    rep["direct_at_r_star"] = chosen_r_cells(w, gpu["S"], gpu["r_idx"], RTOL["exact"], 18)
     print(rep)
 
 
@@ -79,7 +109,8 @@ def test_lognormal_k8_n1e5_fp64_full_grid():
     w = lognormal_workload_k8_n1e5()
     gpu = run(w, kvdro.KVDRO_FP64)
     rep = compare_full(w, gpu, oracle_from_S(w, O.envelope_grid(w)), "fp64")
-    rep["direct"] = direct_cells(w, gpu["S"], 1024, RTOL["fp64"], 2)
+    rep["direct"] = direct_cells(w, gpu["S"], 4096, RTOL["fp64"], 2)
+    rep["direct_at_r_star"] = chosen_r_cells(w, gpu["S"], gpu["r_idx"], RTOL["fp64"], 12)
     print(rep)
 
 
@@ -87,7 +118,8 @@ def test_heavy_tail_k16_n1e6_fp32_full_grid():
     w = heavy_tail_workload_k16_n1e6()
     gpu = run(w, kvdro.KVDRO_FP32)
     rep = compare_full(w, gpu, oracle_from_S(w, O.envelope_grid(w)), "fp32")
-    rep["direct"] = direct_cells(w, gpu["S"], 256, RTOL["fp32"], 3)
+    rep["direct"] = direct_cells(w, gpu["S"], 4096, RTOL["fp32"], 3)
+    rep["direct_at_r_star"] = chosen_r_cells(w, gpu["S"], gpu["r_idx"], RTOL["fp32"], 13)
     print(rep)
 
 
@@ -99,7 +131,8 @@ def test_regime_sweep_slice_and_critical_fractile():
     gpu = run(w, kvdro.KVDRO_FP32)
     ora = oracle_from_S(w, O.envelope_grid(w))
     compare_full(w, gpu, ora, "fp32")
-    direct_cells(w, gpu["S"], 256, RTOL["fp32"], 4)
+    direct_cells(w, gpu["S"], 4096, RTOL["fp32"], 4)
+    chosen_r_cells(w, gpu["S"], gpu["r_idx"], RTOL["fp32"], 14)
     _critical_fractile_rows(w, gpu["r_idx"], ora["cost"], ora["r_idx"], RTOL["fp32"])
 
 
@@ -152,5 +185,6 @@ def test_drift_loop_k32_n1e6_iteration(iteration):
     w = drift_loop_workload_k32_n1e6(iteration)
     gpu = run(w, kvdro.KVDRO_FP32)
     rep = compare_full(w, gpu, oracle_from_S(w, O.envelope_grid(w)), "fp32")
-    rep["direct"] = direct_cells(w, gpu["S"], 128, RTOL["fp32"], 5 + iteration)
+    rep["direct"] = direct_cells(w, gpu["S"], 4096, RTOL["fp32"], 5 + iteration)
+    rep["direct_at_r_star"] = chosen_r_cells(w, gpu["S"], gpu["r_idx"], RTOL["fp32"], 15 + iteration)
     print(rep)
