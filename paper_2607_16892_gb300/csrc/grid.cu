@@ -788,6 +788,7 @@ __global__ void __launch_bounds__(C::MAXT, C::MINB) k_grid(const GridArgs a) {
 // threshold t, so sum_n max(kappa x_n + d, 0) = kappa (sum - CS[t-1]) + d (N - C[t-1]).
 constexpr int kEnvR = 8;          // r values per CTA
 constexpr int kEnvThreads = 256;
+constexpr int kEnvTable = 4096;   // lam * eps products kept in shared memory when NL * E is at most this
 
 // Order key of a double for the minimum over lam: equal for equal values (-0 is taken as +0) and
 // ordered as the values are for every non-NaN double, so the comparison runs on integers instead
@@ -800,26 +801,39 @@ __device__ __forceinline__ long long order_key(double v) {
 
 // The envelope kernel's epilogue: each thread takes whole (r, eps) pairs and scans lam in
 // ascending order with a strict comparison, so ties keep the lowest index (as cta_epilogue's
-// reduction does); the cost of every lam is lam * eps + S, rounded as there.  One FP64 multiply
-// and one add per (r, eps, lam), no shuffles.
+// reduction does); the cost of every lam is lam * eps + S, rounded as there.  One FP64 add per
+// (r, eps, lam) when the CTA holds the lam * eps products (s_le, [lam][eps]), else a multiply and
+// an add; no shuffles.
 __device__ __forceinline__ void env_epilogue(const GridArgs& a, const double* s_S, const double* s_lam,
-                                             const double* s_eps, int r_cta0, int m, int k) {
+                                             const double* s_eps, const double* s_le, int r_cta0, int m, int k) {
     for (int p = threadIdx.x; p < kEnvR * a.E; p += blockDim.x) {
         const int rl = p / a.E, e = p % a.E;
         const int ri = r_cta0 + rl;
         if (ri >= a.R) continue;
         const double eps = s_eps[e];
         const double* S = s_S + rl * a.NL;
-        double best = __dadd_rn(__dmul_rn(s_lam[0], eps), S[0]);
+        double best = __dadd_rn(s_le ? s_le[e] : __dmul_rn(s_lam[0], eps), S[0]);
         long long best_key = order_key(best);
         int bj = 0;
-        for (int j = 1; j < a.NL; j++) {
-            const double v = __dadd_rn(__dmul_rn(s_lam[j], eps), S[j]);
-            const long long key = order_key(v);
-            if (key < best_key) {
-                best_key = key;
-                best = v;
-                bj = j;
+        if (s_le) {
+            for (int j = 1; j < a.NL; j++) {
+                const double v = __dadd_rn(s_le[j * a.E + e], S[j]);
+                const long long key = order_key(v);
+                if (key < best_key) {
+                    best_key = key;
+                    best = v;
+                    bj = j;
+                }
+            }
+        } else {
+            for (int j = 1; j < a.NL; j++) {
+                const double v = __dadd_rn(__dmul_rn(s_lam[j], eps), S[j]);
+                const long long key = order_key(v);
+                if (key < best_key) {
+                    best_key = key;
+                    best = v;
+                    bj = j;
+                }
             }
         }
         const size_t row = ((size_t)m * a.E + e) * a.K + k;
@@ -845,6 +859,9 @@ __global__ void __launch_bounds__(kEnvThreads) k_envelope(const GridArgs a) {
     for (int i = threadIdx.x; i < a.NL; i += blockDim.x) s_lam[i] = a.lam[i];
     for (int i = threadIdx.x; i < a.E; i += blockDim.x) s_eps[i] = a.eps[i];
     __syncthreads();
+    double* s_le = a.NL * a.E <= kEnvTable ? s_S + kEnvR * a.NL : nullptr;  // [lam][eps] products
+    if (s_le)
+        for (int i = threadIdx.x; i < a.NL * a.E; i += blockDim.x) s_le[i] = __dmul_rn(s_lam[i / a.E], s_eps[i % a.E]);
     const double cp = a.cp[m], cw = a.cw[m];
     const int32_t Lk = a.L[k];
     const int64_t Nk = a.N[k];
@@ -869,7 +886,7 @@ __global__ void __launch_bounds__(kEnvThreads) k_envelope(const GridArgs a) {
         if (a.S_out) static_cast<double*>(a.S_out)[(((size_t)m * a.K + k) * a.R + ri) * a.NL_out + a.lam0 + j] = S;
     }
     __syncthreads();
-    env_epilogue(a, s_S, s_lam, s_eps, r_cta0, m, k);
+    env_epilogue(a, s_S, s_lam, s_eps, s_le, r_cta0, m, k);
 }
 
 template <Prec P>
@@ -918,7 +935,7 @@ GridShape grid_shape(Prec p, int32_t R, int32_t NL, int32_t E, int32_t max_L) {
         sh.RG = 1;
         sh.threads = kEnvThreads;
         sh.r_blocks = (R + kEnvR - 1) / kEnvR;
-        sh.smem = 8 * ((size_t)NL + E + (size_t)kEnvR * NL);
+        sh.smem = 8 * ((size_t)NL + E + (size_t)kEnvR * NL + ((int64_t)NL * E <= kEnvTable ? (size_t)NL * E : 0));
         return sh;
     }
     if (p == Prec::F64) return shape_for<CfgF64>(2, R, NL, E);
@@ -944,7 +961,7 @@ cudaError_t grid_prepare(Prec p) {
     }
     if (p == Prec::ENVELOPE)
         return cudaFuncSetAttribute(k_envelope, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    (int)(8 * (256 + 64 + (size_t)kEnvR * 256)));
+                                    (int)(8 * (256 + 64 + (size_t)kEnvR * 256 + kEnvTable)));
     cudaError_t e = cudaFuncSetAttribute(k_grid<CfgF32>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
     if (e != cudaSuccess) return e;
     return cudaFuncSetAttribute(k_grid<CfgF32Wide>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
