@@ -570,3 +570,44 @@ def test_exact_sums_stay_exact_at_the_fold_bound(L):
     np.testing.assert_allclose(ex["S"], env["S"], rtol=1e-12, atol=0)
     compare_full(w, ex, O.solve(w), "exact")
     compare_full(w, run(w, P["fp32"]), O.solve(w), "fp32")
+
+
+@pytest.mark.parametrize("L", [900, 1 << 20, (1 << 22) + 3])
+def test_class_sizes_at_chunk_and_padding_boundaries(L):
+    """Classes whose sizes sit on and around the staged chunk sizes (6144 samples in the exact
+    kernels, 4096 in the FP32 and FP64 ones) and the 128-sample padding unit, one sample each side:
+    the fast full-chunk path, the ragged last chunk and the padded tail all meet the oracle.  The
+    supports select the mixed exact kernel (900), the all-integer one (2^20) and, above 2^22, the
+    FP32-arithmetic kernel for FP32 requests."""
+    rng = np.random.default_rng(L)
+    sizes = (1, 127, 128, 129, 4095, 4096, 4097, 6143, 6144, 6145, 12288, 12289)
+    cls = [np.minimum(L, rng.integers(0, min(L, 5000) + 1, n)) for n in sizes]
+    w = make(cls, L, np.unique(np.linspace(0, L, 11).astype(np.int64)), [0.02, 0.5, 1.0, 4.0, 30.0], [0.0, 7.0, 90.0],
+             [6.0, 1.0], [1.0, 3.0], name=f"sizes{L}")
+    ref = O.solve(w)
+    modes = ["fp32", "fp64"] + (["exact"] if L <= (1 << 22) else [])
+    for mode in modes:
+        compare_full(w, run(w, P[mode]), ref, mode)
+
+
+def test_a_wait_that_runs_out_with_regime_blocks_of_host_outputs(monkeypatch):
+    """The bounded-wait test hook with several regimes and host outputs, which come back in regime
+    blocks on the context's copy stream: the call still reports KVDRO_ETIMEOUT once every copy is
+    done, and the device then evaluates correctly."""
+    rng = np.random.default_rng(9)
+    w = make([rng.integers(0, 900, 20000), rng.integers(0, 700, 3000)], 1000, [10, 200, 600], [0.5, 5.0],
+             [0.0, 10.0], [10.0, 3.0, 1.5], [1.0, 1.0, 2.0])
+    monkeypatch.setenv("KVDRO_TEST_SKIP_CHUNK", "1")
+    ctx = kvdro.kvdro_create(0)
+    monkeypatch.delenv("KVDRO_TEST_SKIP_CHUNK")
+    try:
+        kvdro.kvdro_load_samples(ctx, w.K, w.offsets, torch.from_numpy(w.samples).cuda(), w.L, w.L_in)
+        M, E, K, R = len(w.cp), len(w.eps), w.K, len(w.r)
+        out = {"cost": np.empty((M, E, K, R), np.float32), "lam_idx": np.empty((M, E, K, R), np.int32),
+               "r_idx": np.empty((M, E, K), np.int32)}
+        st = _status(kvdro.kvdro_eval_grid, ctx, P["fp32"], R, w.r, 2, w.lam, E, w.eps, M, w.cp, w.cw, **out)
+        assert st == kvdro.KVDRO_ETIMEOUT
+        assert "gave up waiting" in kvdro.kvdro_last_error(ctx)
+    finally:
+        kvdro.kvdro_destroy(ctx)
+    compare_full(w, run(w, P["fp32"], host_outputs=True), O.solve(w), "fp32")
