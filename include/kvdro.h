@@ -119,8 +119,10 @@ int kvdro_quantiles(kvdro_ctx* ctx, int32_t F, const double* fractiles, int32_t*
  *   E, eps     host double[E], finite, >= 0; 1 <= E <= 64.
  *   M, c_p,c_w host double[M] each, finite, >= 0; 1 <= M <= 65536.
  * Outputs (each may be NULL to skip it; host or device).  With M > 1, host S, cost and lam_idx
- * come back in up to 16 blocks of regimes on a stream of the context's own, each block's copy
- * overlapping the evaluation of the next; the call still returns only once every output is filled.
+ * come back in up to 16 blocks of regimes on a stream of the context's own; into page-locked host
+ * memory each block's copy overlaps the evaluation of the next (a copy into pageable memory holds
+ * the calling thread until it is done, so those blocks alternate with the evaluation instead).
+ * The call returns only once every output is filled.
  *   S          [M][K][R][NL]  mean supremum S(eta, lam)
  *   cost       [M][E][K][R]   min over lam of lam*eps + S
  *   lam_idx    int32 [M][E][K][R]  lowest lam index attaining cost
